@@ -1,0 +1,32 @@
+"""CPU oracle for the dual-sparse batch-1 spMspV of DuoGPT (arXiv 2506.20194).
+
+TEST INFRASTRUCTURE ONLY.  Nothing in the product path imports this package:
+only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` may import or call it.  It shares no
+code with the CUDA library (no kernels, headers, tables or helpers) and does
+not import ``paper_2506_20194_gb300``.
+
+Every function is pinned by ``tests/test_oracle_*.py`` against something other
+than itself (exact integer arithmetic, exactly-rounded summation, brute force
+on tiny inputs, closed forms and invariants).  No function here is "parity
+unpinned".
+"""
+from .duo_oracle import (  # noqa: F401
+    SEG_ROWS,
+    CMB_MAGIC,
+    IDX16_MAGIC,
+    k_from_pct,
+    oracle_sparsify,
+    oracle_spmspv,
+    oracle_spmspv_rows,
+    exact_spmspv_rows_scaled,
+    fsum_spmspv_rows,
+    tolerance_rows,
+    ref_pack_cmb,
+    ref_unpack_cmb,
+    ref_pack_idx16,
+    ref_unpack_idx16,
+    required_bytes,
+    loaded_fraction,
+    worst_case_loaded_fraction,
+)
