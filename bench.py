@@ -1,0 +1,516 @@
+"""Benchmark: batch-1 dual-sparse spMspV over a LLaMA-2-7B-shaped decoder layer.
+
+One step = one decoder layer's seven projections at 50% weight / 50%
+activation sparsity, launched as a decode step must order them: the fused
+sparsify + spMspV of q/k/v (one shared input), then o, then gate/up (one
+shared input), then down (four launches of the CUDA kernel).  Eight distinct
+seeded layers rotate so that every step streams weights that are not in L2.
+
+Printed metric: effective HBM GB/s on the required bytes (the kept channels'
+fp16 non-zeros, one mask bit per kept position, x, kept ids/values and y),
+plus microseconds per layer.  See the design doc for the byte model.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "µs/layer and effective HBM GB/s (% of GB300 peak) for batch-1 dual-sparse spMspV"
+WORKLOAD = "llama2-7b-layer"
+STAGES = (("q", "k", "v"), ("o",), ("gate", "up"), ("down",))
+STAGE_SRC = ("q", "o", "gate", "down")
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=16000)
+    ap.add_argument("--warmup", type=int, default=400)
+    ap.add_argument("--impl", default="ours", choices=("ours", "reference"))
+    ap.add_argument("--layers", type=int, default=8, help="distinct layers rotated")
+    ap.add_argument("--px", type=int, default=50)
+    ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--profile", action="store_true",
+                    help="small case for ncu: 2 layers, a few direct (ungraphed) layer steps")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------- helpers --
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi sampling during the timed region (clocks, throttle reasons)."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, smax, reasons = [], None, set()
+        names = ("active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names[1:], parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": smax,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def make_layers(duo, synth, L, device, px):
+    """Packs L distinct LLaMA-2-7B-shaped layers; returns per-layer dicts."""
+    wl = synth.WORKLOADS[WORKLOAD]
+    shape = wl["shape"]
+    layers = []
+    for l in range(L):
+        Ws = {p: synth.layer_weight(wl, p, layer=l, device=device) for p in synth.PROJS}
+        hs = {p: duo.duo_pack(Ws[p], "bitmask") for p in synth.PROJS}
+        nnz = {p: (Ws[p] != 0).sum(dim=0).to(torch.int64) for p in synth.PROJS}
+        xs = {s: synth.layer_input(wl, s, layer=l, device=device) for s in STAGE_SRC}
+        ys = {p: torch.empty(shape.O(p), dtype=torch.float32, device=device) for p in synth.PROJS}
+        layers.append(dict(W=Ws, h=hs, nnz=nnz, x=xs, y=ys))
+    return shape, layers
+
+
+def k_of(I, px):
+    return (I * (100 - px)) // 100
+
+
+def required_bytes_layer(duo, shape, layer, px):
+    """Format-neutral required bytes of one layer step, with the kept sets
+    taken from the library's own (parity-tested) sparsifier."""
+    total = 0.0
+    per_stage = []
+    for st, src in zip(STAGES, STAGE_SRC):
+        I = shape.I(st[0])
+        k = k_of(I, px)
+        b = 0.0
+        if k > 0:
+            idx, _ = duo.duo_sparsify(layer["x"][src], k)
+            K = idx.to(torch.int64) & 0xFFFF
+        for p in st:
+            O = shape.O(p)
+            vals = float(layer["nnz"][p][K].sum().item()) * 2.0 if k > 0 else 0.0
+            b += vals + k * O / 8.0 + 4.0 * O
+        b += 2.0 * I + 4.0 * k
+        per_stage.append(b)
+        total += b
+    return total, per_stage
+
+
+def stage_calls(duo, shape, layer, px):
+    def run():
+        for st, src in zip(STAGES, STAGE_SRC):
+            k = k_of(shape.I(st[0]), px)
+            if len(st) == 1:
+                duo.duo_spmspv(layer["h"][st[0]], layer["x"][src], k, y=layer["y"][st[0]])
+            else:
+                duo.duo_spmspv_multi([layer["h"][p] for p in st], layer["x"][src], k,
+                                     ys=[layer["y"][p] for p in st])
+    return run
+
+
+def capture_rotation(duo, shape, layers, px, with_events):
+    """One CUDA graph replaying every layer once (L steps), with timing
+    events around each stage launch when supported."""
+    events = None
+    if with_events:
+        try:
+            events = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(len(STAGES) + 1)]
+                      for _ in layers]
+        except TypeError:
+            events = None
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):           # warm the launch path (attributes, module load)
+        for layer in layers:
+            stage_calls(duo, shape, layer, px)()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for li, layer in enumerate(layers):
+            for si, (st, src) in enumerate(zip(STAGES, STAGE_SRC)):
+                if events is not None:
+                    events[li][si].record()
+                k = k_of(shape.I(st[0]), px)
+                if len(st) == 1:
+                    duo.duo_spmspv(layer["h"][st[0]], layer["x"][src], k, y=layer["y"][st[0]])
+                else:
+                    duo.duo_spmspv_multi([layer["h"][p] for p in st], layer["x"][src], k,
+                                         ys=[layer["y"][p] for p in st])
+            if events is not None:
+                events[li][len(STAGES)].record()
+    return g, events
+
+
+def time_graph(g, reps):
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(reps):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) * 1e-3
+
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(v, world):
+    if world == 1:
+        return v
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --------------------------------------------------------- CPU oracle arm --
+
+def oracle_layer_sample(shape, cpu_layer, px, row_frac):
+    """Runs the oracle on a row sample of every projection of one layer;
+    returns (seconds, required bytes covered by the sample)."""
+    import oracle as orc
+    t0 = time.perf_counter()
+    covered = 0.0
+    for st, src in zip(STAGES, STAGE_SRC):
+        x16 = cpu_layer["x"][src]
+        I = x16.size
+        k = k_of(I, px)
+        for p in st:
+            W = cpu_layer["W"][p]
+            O = W.shape[0]
+            nr = max(1, int(round(O * row_frac)))
+            y = orc.oracle_spmspv_rows(W[:nr], x16, k)
+            assert y.shape[0] == nr
+            covered += cpu_layer["breq"][p] * nr / O
+    return time.perf_counter() - t0, covered
+
+
+def cpu_layer_from(layer, shape, px):
+    """Host copies of one layer (fp16 numpy) plus per-projection required bytes."""
+    W = {p: layer["W"][p].cpu().numpy().view(np.float16) for p in layer["W"]}
+    x = {s: layer["x"][s].cpu().numpy().view(np.float16) for s in STAGE_SRC}
+    import oracle as orc
+    breq = {}
+    for st, src in zip(STAGES, STAGE_SRC):
+        I = shape.I(st[0])
+        k = k_of(I, px)
+        K, _ = orc.oracle_sparsify(x[src], k)
+        for p in st:
+            nnz = (W[p] != 0).sum(axis=0)
+            breq[p] = orc.required_bytes(nnz, K, shape.O(p), I)
+    return dict(W=W, x=x, breq=breq)
+
+
+def cpu_baseline(shape, layer, px, seconds):
+    cl = cpu_layer_from(layer, shape, px)
+    # calibrate a row fraction so that one sample step takes ~0.5 s
+    t, cov = oracle_layer_sample(shape, cl, px, 1.0 / 64)
+    frac = min(1.0, (1.0 / 64) * 0.5 / max(t, 1e-6))
+    tot_t, tot_b, n = 0.0, 0.0, 0
+    while tot_t < seconds:
+        t, cov = oracle_layer_sample(shape, cl, px, frac)
+        tot_t += t
+        tot_b += cov
+        n += 1
+    gbs = tot_b / tot_t / 1e9
+    full_layer_b = sum(cl["breq"].values())
+    return {"value": gbs, "unit": "GB/s", "cores": os.cpu_count(), "kind": "oracle",
+            "us_per_layer": full_layer_b / (gbs * 1e9) * 1e6,
+            "sample": f"{n} steps of the fp64 numpy oracle on {frac:.4f} of every projection's rows "
+                      f"of one {WORKLOAD} (px={px}), {tot_t:.1f} s; numpy BLAS threads default "
+                      f"(all {os.cpu_count()} cores)"}
+
+
+def run_reference(args):
+    world, rank, _ = dist_setup(args)
+    if rank != 0:
+        return
+    from paper_2506_20194_gb300 import synth
+    wl = synth.WORKLOADS[WORKLOAD]
+    shape = wl["shape"]
+    layer = {"W": {p: synth.layer_weight(wl, p, layer=0) for p in synth.PROJS},
+             "x": {s: synth.layer_input(wl, s, layer=0) for s in STAGE_SRC}}
+    cl = cpu_layer_from(layer, shape, args.px)
+    t, _ = oracle_layer_sample(shape, cl, args.px, 1.0 / 256)
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    frac = min(1.0, max(1.0 / 4096, (1.0 / 256) * budget / max(t, 1e-6)))
+    for _ in range(args.warmup):
+        oracle_layer_sample(shape, cl, args.px, frac)
+    tot_t, tot_b = 0.0, 0.0
+    for _ in range(args.steps):
+        t, cov = oracle_layer_sample(shape, cl, args.px, frac)
+        tot_t += t
+        tot_b += cov
+    gbs = tot_b / tot_t / 1e9
+    sample = (f"fp64 numpy oracle on {frac:.5f} of every projection's rows of one {WORKLOAD} "
+              f"layer per step (px={args.px})")
+    line = {"impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": tot_t / max(1, args.steps) * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "px": args.px, "pw": 0.5},
+            "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": os.cpu_count(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------- our arm --
+
+def run_ours(args):
+    world, rank, local = dist_setup(args)
+    assert torch.cuda.is_available(), "bench.py needs a CUDA device"
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2506_20194_gb300 import duo, synth
+    duo.load_library()
+    L = args.layers
+    shape, layers = make_layers(duo, synth, L, dev, args.px)
+    breq_layers = [required_bytes_layer(duo, shape, lay, args.px) for lay in layers]
+    breq_mean = float(np.mean([b for b, _ in breq_layers]))
+    stage_b = np.mean(np.array([ps for _, ps in breq_layers]), axis=0)
+
+    g, events = capture_rotation(duo, shape, layers, args.px, with_events=True)
+    reps_w = max(1, math.ceil(args.warmup / L))
+    reps = max(1, args.steps // L)
+    steps_timed = reps * L
+    time_graph(g, reps_w)
+    sampler = ClockSampler(local)
+    barrier(world)
+    sampler.start()
+    t = time_graph(g, reps)
+    clocks = sampler.stop()
+    barrier(world)
+    t = max_over_ranks(t, world)
+    assert duo.duo_device_status() == duo.DUO_OK
+    us_layer = t / steps_timed * 1e6
+    value = breq_mean * steps_timed * world / t / 1e9
+
+    # per-stage kernel durations from the in-graph events of the last replay
+    stage_us = None
+    if events is not None:
+        try:
+            st_ms = np.array([[events[l][s].elapsed_time(events[l][s + 1]) for s in range(len(STAGES))]
+                              for l in range(L)])
+            stage_us = st_ms.mean(axis=0) * 1e3
+        except Exception:
+            stage_us = None
+    peak, peak_kind = peaks()
+    if stage_us is not None:
+        achieved = float(stage_b.sum() / (stage_us.sum() * 1e-6) / 1e9)
+    else:
+        achieved = breq_mean / (us_layer * 1e-6) / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "peak_kind": peak_kind, "traffic": None,
+                "kernel": "cmb_spmspv_kernel<fused>",
+                "per_launch_bytes": [float(b) for b in stage_b],
+                "per_launch_us": None if stage_us is None else [float(u) for u in stage_us]}
+
+    # end to end through the public API with host buffers
+    e2e = run_e2e(duo, shape, layers, args, breq_mean)
+
+    # dense fp16 GEMV (cuBLAS via F.linear) over the same rotation
+    dense = run_dense(shape, layers, reps=max(1, min(reps, 200)))
+
+    sweep = {}
+    if not args.no_sweep:
+        for px in (0, 25, 50, 70):
+            gs, _ = capture_rotation(duo, shape, layers, px, with_events=False)
+            time_graph(gs, 5)
+            r = max(1, min(reps, 400))
+            ts = time_graph(gs, r)
+            b = float(np.mean([required_bytes_layer(duo, shape, lay, px)[0] for lay in layers]))
+            us = ts / (r * L) * 1e6
+            sweep[str(px)] = {"us_per_layer": us, "GB/s": b / (us * 1e-6) / 1e9,
+                              "frac_of_peak": b / (us * 1e-6) / 1e9 / peak, "required_MB": b / 1e6}
+            del gs
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(shape, layers[0], args.px, args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "GB/s", "us_per_layer": us_layer,
+            "n_gpus": world, "steps": steps_timed, "warmup": reps_w * L,
+            "ms_per_step": us_layer * 1e-3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "shapes": "q/k/v/o 4096x4096, gate/up 11008x4096, down 4096x11008",
+                       "pw": 0.5, "prune": "magnitude, exact count per 128-channel block",
+                       "px": args.px, "format": "bitmask (CMB)", "layers_rotated": L,
+                       "l2": f"inputs larger than L2: {L} distinct packed layers rotated",
+                       "required_MB_per_layer": breq_mean / 1e6, "parallelism": "replicas" if world > 1 else "1gpu"},
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": steps_timed * len(STAGES),
+            "clocks": clocks,
+            "dense_gemv_cublas": dense,
+            "sweep_px": sweep,
+        }
+        print(json.dumps(line), flush=True)
+    for lay in layers:
+        for h in lay["h"].values():
+            h.free()
+
+
+def run_e2e(duo, shape, layers, args, breq_mean):
+    """Public-API calls with host (pinned) inputs copied in and outputs read
+    back every step; no graph (this is the call a user makes)."""
+    L = len(layers)
+    hx = [{s: layers[l]["x"][s].cpu().pin_memory() for s in STAGE_SRC} for l in range(L)]
+    hy = [{p: torch.empty(shape.O(p), dtype=torch.float32).pin_memory() for p in layers[l]["y"]}
+          for l in range(L)]
+    h2d = sum(t.numel() * 2 for t in hx[0].values())
+    d2h = sum(t.numel() * 4 for t in hy[0].values())
+
+    def step(i):
+        l = i % L
+        lay = layers[l]
+        for s in STAGE_SRC:
+            lay["x"][s].copy_(hx[l][s], non_blocking=True)
+        stage_calls(duo, shape, lay, args.px)()
+        for p in lay["y"]:
+            hy[l][p].copy_(lay["y"][p], non_blocking=True)
+
+    n = min(args.steps, 2000)
+    for i in range(min(args.warmup, 50)):
+        step(i)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(n):
+        step(i)
+    torch.cuda.synchronize()
+    t = time.perf_counter() - t0
+    return {"value": breq_mean * n / t / 1e9, "unit": "GB/s", "us_per_layer": t / n * 1e6,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n}
+
+
+def run_dense(shape, layers, reps):
+    L = len(layers)
+    xs = [{p: layers[l]["x"][{"k": "q", "v": "q", "up": "gate"}.get(p, p)] for p in layers[l]["W"]}
+          for l in range(L)]
+    outs = [{p: torch.empty(shape.O(p), dtype=torch.float16, device=layers[0]["x"]["q"].device)
+             for p in layers[l]["W"]} for l in range(L)]
+
+    def run():
+        for l in range(L):
+            for p, W in layers[l]["W"].items():
+                torch.matmul(W, xs[l][p], out=outs[l][p])
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        run()
+    torch.cuda.current_stream().wait_stream(s)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        run()
+    time_graph(g, 3)
+    t = time_graph(g, reps)
+    us = t / (reps * L) * 1e6
+    dense_bytes = sum(W.numel() * 2 + W.shape[1] * 2 + W.shape[0] * 2 for W in layers[0]["W"].values())
+    return {"us_per_layer": us, "GB/s": dense_bytes / (us * 1e-6) / 1e9, "bytes_per_layer": dense_bytes}
+
+
+def run_profile(args):
+    """Small workload for profiler captures: packs 2 layers and runs
+    `--steps` layer steps (4 fused spMspV launches each) without graphs."""
+    torch.cuda.set_device(0)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2506_20194_gb300 import duo, synth
+    duo.load_library()
+    shape, layers = make_layers(duo, synth, 2, torch.device("cuda", 0), args.px)
+    for i in range(args.steps):
+        stage_calls(duo, shape, layers[i % 2], args.px)()
+    torch.cuda.synchronize()
+    assert duo.duo_device_status() == duo.DUO_OK
+    print("profile workload done", flush=True)
+
+
+def main():
+    args = parse()
+    if args.profile:
+        run_profile(args)
+    elif args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,190 @@
+/*
+ * duo.h -- C ABI of the GB300 (sm_103a) dual-sparse batch-1 spMspV library.
+ *
+ * The library computes the decode-time product of DuoGPT (arXiv 2506.20194),
+ * §3 "Activation Sparsity":
+ *
+ *     y = W (x ⊙ m^x) = sum_{i : m^x_i = 1} W[:, i] * x_i
+ *
+ * where W (O rows x I input channels, fp16) carries unstructured weight
+ * sparsity (pruned entries are stored as zero, §3 mask m^w) and m^x keeps the
+ * k input channels of largest |x_i|, chosen "on the fly" (§3).  §4.1
+ * describes the execution: only the compressed weight columns of the
+ * surviving channels are fetched from HBM.
+ *
+ * Conventions shared by every entry point:
+ *   - Every call returns an int status (DUO_OK or a negative DUO_E* code) and
+ *     never aborts the process.  Arguments are validated on the host before
+ *     any CUDA call; an invalid call changes nothing.
+ *   - Pointers named *_dev are device pointers of the current CUDA device;
+ *     the caller owns them (typically PyTorch tensors) and keeps them alive
+ *     until the work enqueued on `stream` has finished.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Calls documented "async" only enqueue work on it.
+ *   - Channel ids are uint16, so I <= 65535.
+ *   - Device-side waits are bounded; a wait that runs out sets a device
+ *     status word that duo_device_status() returns (DUO_ETIMEOUT).
+ *   - There is no host fallback: without a usable CUDA device every compute
+ *     entry point returns DUO_ECUDA.
+ */
+#ifndef DUO_H
+#define DUO_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DUO_ABI_VERSION 1
+
+/* Status codes. */
+enum {
+    DUO_OK = 0,
+    DUO_EINVAL = -1,    /* bad argument: NULL, size, alignment, dead handle */
+    DUO_ENOMEM = -2,    /* device allocation failed (nothing leaked) */
+    DUO_ECUDA = -3,     /* a CUDA runtime call failed or no device */
+    DUO_ERANGE = -4,    /* a size exceeds what the format can index */
+    DUO_EFORMAT = -5,   /* handle format does not support the call */
+    DUO_ETIMEOUT = -6   /* a bounded device-side wait ran out */
+};
+
+/* Packed weight formats (the paper fixes none: §4.1 only says each weight
+ * column is stored compressed; both layouts below are this library's). */
+enum {
+    DUO_FMT_IDX16 = 0,   /* per channel: fp16 non-zeros + uint16 row ids */
+    DUO_FMT_BITMASK = 1  /* "CMB": per (channel, 1024-row segment) a 128-byte
+                            row bitmask followed by the fp16 non-zeros */
+};
+
+/* Opaque packed weight, owned by the library from duo_pack to duo_free. */
+typedef struct duo_packed duo_packed;
+
+/*
+ * duo_pack -- compress a pruned weight into channel-major storage
+ * (§4.1: "only the compressed model parameters are loaded"; §3 footnote:
+ * weights are stored column-major, i.e. one run per input channel).
+ *
+ *   W_fp16_dev : device, fp16, row-major O x I with leading dimension ldw
+ *                (element (r, j) at W[r * ldw + j]); entries equal to +0 or
+ *                -0 are pruned, every other entry is stored bit-exactly.
+ *   out, in    : O >= 1 and 1 <= I <= 65535; IDX16 also needs O <= 65536.
+ *   ldw        : >= in.
+ *   fmt        : DUO_FMT_BITMASK or DUO_FMT_IDX16.
+ *   stream     : work is enqueued on it and the call synchronises it before
+ *                returning (the packed size must be known to allocate).
+ *   h_out      : receives the new handle; untouched on error.
+ *
+ * BITMASK layout (normative): S = ceil(O / 1024) row segments; for input
+ * channel j (outer) and segment s (inner) a record at byte 16 * off[j*S + s]
+ * of the data buffer: 32 little-endian uint32 mask words (bit b of word w set
+ * iff W[s*1024 + 32*w + b, j] != 0; rows >= O give 0), then those entries'
+ * fp16 bit patterns in increasing row order, zero padded to 16 bytes.
+ * off is uint32[I*S + 1]; off[I*S] is the total size in 16-byte units.
+ *
+ * IDX16 layout: per channel j a block at byte colptr[j]: cnt[j] fp16
+ * non-zeros (increasing row), zero padded to 16 bytes, then their uint16 row
+ * ids, zero padded to 16 bytes.  colptr is uint64[I + 1], cnt is uint32[I].
+ *
+ * Errors: DUO_EINVAL (NULL, sizes, ldw, fmt), DUO_ERANGE (format limits),
+ * DUO_ENOMEM, DUO_ECUDA.
+ */
+int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw,
+             int fmt, void* stream, duo_packed** h_out);
+
+/*
+ * duo_sparsify -- the activation mask of §3: keep the k channels of largest
+ * |x_i| (equal magnitudes: the lower index is kept first; +0 and -0 have
+ * magnitude 0; NaN orders above Inf by bit pattern).  Async.
+ *
+ *   x_fp16_dev        : device, fp16[in].
+ *   in                : 1..65535.   k : 0..in.
+ *   kept_idx_dev      : device, uint16[k]: the kept channel ids, ascending.
+ *   kept_val_fp16_dev : device, fp16[k]: x at those ids, bit-exact.
+ * Errors: DUO_EINVAL, DUO_ECUDA.
+ */
+int duo_sparsify(const void* x_fp16_dev, int64_t in, int64_t k,
+                 uint16_t* kept_idx_dev, void* kept_val_fp16_dev, void* stream);
+
+/*
+ * duo_spmspv -- y = W (x ⊙ m^x) over the packed weight (§3, §4.1).  Async.
+ *
+ * Two modes:
+ *   fused   : kept_idx_dev == kept_val_fp16_dev == NULL.  The kernel selects
+ *             the k largest-|x| channels itself (same rule as duo_sparsify)
+ *             from x_fp16_dev (device fp16[in]) and streams only their
+ *             compressed columns.
+ *   listed  : kept_idx_dev (uint16[k], distinct ids < in, any order) and
+ *             kept_val_fp16_dev (fp16[k]) give the sparse input directly;
+ *             x_fp16_dev is ignored and may be NULL.
+ *   y_dev   : device fp32[O], 16-byte aligned; fully overwritten (the call
+ *             zeroes it on `stream` first).  Summation order is not fixed,
+ *             so y is reproducible only to fp32 rounding.
+ * Errors: DUO_EINVAL (NULL, alignment, k, dead handle), DUO_ECUDA.
+ */
+/* Concurrency: calls whose first handle is the same must be ordered on the
+ * GPU (same stream, or otherwise synchronised): the bitmask kernel keeps a
+ * small grid-barrier state with that handle. */
+int duo_spmspv(const duo_packed* h, const void* x_fp16_dev,
+               const uint16_t* kept_idx_dev, const void* kept_val_fp16_dev,
+               int64_t k, float* y_dev, void* stream);
+
+/*
+ * duo_spmspv_multi -- n (1..4) products that share one sparse input, in one
+ * launch and with one selection: y_p = W_p (x ⊙ m^x) for p < n.  In a
+ * decoder layer the q/k/v projections read the same input, as do gate/up
+ * (the per-layer linear layers of §5's LLaMA models).  All handles must be
+ * DUO_FMT_BITMASK with the same I; O may differ.  Arguments as in
+ * duo_spmspv, with ys_dev[p] the output of handle hs[p].  Async.
+ */
+int duo_spmspv_multi(const duo_packed* const* hs, int n, const void* x_fp16_dev,
+                     const uint16_t* kept_idx_dev, const void* kept_val_fp16_dev,
+                     int64_t k, float* const* ys_dev, void* stream);
+
+/* duo_free -- release a handle and its device memory.  NULL is a no-op
+ * (DUO_OK); a handle that is not live (already freed, never created)
+ * returns DUO_EINVAL without touching memory.  Synchronises the device
+ * memory release with cudaFree semantics. */
+int duo_free(duo_packed* h);
+
+/* Describes a live handle.  Pointers stay owned by the handle.
+ *   BITMASK: index = uint32 off[I*S+1], aux = NULL.
+ *   IDX16  : index = uint64 colptr[I+1], aux = uint32 cnt[I]. */
+typedef struct duo_packed_info {
+    int32_t fmt;
+    int32_t version;
+    uint32_t magic;          /* "CMB1" or "IDX0" little-endian */
+    int32_t seg_rows;        /* 1024 for BITMASK, 0 for IDX16 */
+    int64_t out, in, nseg, nnz;
+    const void* index_dev; int64_t index_bytes;
+    const void* aux_dev;   int64_t aux_bytes;
+    const void* data_dev;  int64_t data_bytes;
+} duo_packed_info;
+
+int duo_packed_query(const duo_packed* h, duo_packed_info* info);
+
+/* Copies one buffer of a live handle to host memory (synchronous), e.g. to
+ * save a packed weight or to compare its bytes with a reference packer.
+ *   which : 0 = index, 1 = aux, 2 = data (as described by duo_packed_info).
+ *   dst_host, bytes : host destination; bytes must equal the buffer size.
+ * Errors: DUO_EINVAL (dead handle, which, NULL dst, size mismatch), DUO_ECUDA. */
+int duo_packed_export(const duo_packed* h, int which, void* dst_host, int64_t bytes);
+
+/* Synchronises `stream`, returns and clears the device status word:
+ * DUO_OK; DUO_ETIMEOUT if a bounded device wait ran out since the last
+ * call; DUO_EFORMAT if a kernel met a record size or channel id outside the
+ * format's bounds (the affected work was skipped); DUO_ECUDA if the stream
+ * reports an error. */
+int duo_device_status(void* stream);
+
+/* Text of a status code (static storage). */
+const char* duo_strerror(int code);
+
+/* DUO_ABI_VERSION of the loaded library. */
+int duo_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DUO_H */

@@ -1,0 +1,411 @@
+// C ABI of libduo (include/duo.h): argument validation, handle ownership and
+// launch dispatch.  Host code only; every kernel lives in kernels.cu.
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <unordered_set>
+
+#include <cuda_runtime.h>
+
+#include "../../include/duo.h"
+#include "duo_launch.h"
+
+namespace {
+
+constexpr uint32_t kHandleMagic = 0x4455504Bu;  // "KPUD"
+constexpr uint32_t kCmbMagic = 0x31424D43u;     // "CMB1"
+constexpr uint32_t kIdx16Magic = 0x30584449u;   // "IDX0"
+
+}  // namespace
+
+struct duo_packed {
+  uint32_t magic;
+  int fmt;
+  int device;
+  int64_t out, in, nseg, nnz;
+  void* index;
+  int64_t index_bytes;
+  void* aux;
+  int64_t aux_bytes;
+  void* data;
+  int64_t data_bytes;
+  unsigned int* sync;  // BITMASK: 2-word grid barrier of the spMspV kernel
+};
+
+namespace {
+
+std::mutex g_mu;
+std::unordered_set<const duo_packed*>& live_handles() {
+  static std::unordered_set<const duo_packed*> s;
+  return s;
+}
+
+bool is_live(const duo_packed* h) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  return live_handles().count(h) != 0 && h->magic == kHandleMagic;
+}
+
+int map_err(cudaError_t e) {
+  if (e == cudaSuccess) return DUO_OK;
+  if (e == cudaErrorMemoryAllocation) return DUO_ENOMEM;
+  return DUO_ECUDA;
+}
+
+// Allocation with an optional injected failure: DUO_FAULT_ALLOC_FAIL=n makes
+// the n-th device allocation of the process fail (host-side fault
+// injection for the error paths; no GPU fault is involved).
+std::mutex g_alloc_mu;
+long g_alloc_count = 0;
+long fault_alloc_target() {
+  static long target = [] {
+    const char* s = std::getenv("DUO_FAULT_ALLOC_FAIL");
+    return s ? std::atol(s) : 0L;
+  }();
+  return target;
+}
+
+cudaError_t duo_malloc(void** p, size_t bytes) {
+  {
+    std::lock_guard<std::mutex> lk(g_alloc_mu);
+    ++g_alloc_count;
+    const long t = fault_alloc_target();
+    if (t > 0 && g_alloc_count == t) {
+      *p = nullptr;
+      return cudaErrorMemoryAllocation;
+    }
+  }
+  return cudaMalloc(p, bytes == 0 ? 16 : bytes);
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// True if p is device (or managed) memory of the current context.
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+int cuda_ready() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return DUO_ECUDA;
+  }
+  int n = 0;
+  if (cudaGetDeviceCount(&n) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    return DUO_ECUDA;
+  }
+  return DUO_OK;
+}
+
+struct Scratch {
+  void* p[8] = {};
+  int n = 0;
+  void* add(void* q) { p[n++] = q; return q; }
+  ~Scratch() {
+    for (int i = 0; i < n; ++i) cudaFree(p[i]);
+  }
+};
+
+}  // namespace
+
+extern "C" {
+
+int duo_abi_version(void) { return DUO_ABI_VERSION; }
+
+const char* duo_strerror(int code) {
+  switch (code) {
+    case DUO_OK: return "ok";
+    case DUO_EINVAL: return "invalid argument";
+    case DUO_ENOMEM: return "device allocation failed";
+    case DUO_ECUDA: return "CUDA runtime error or no usable device";
+    case DUO_ERANGE: return "size exceeds the format's range";
+    case DUO_EFORMAT: return "handle format does not support this call";
+    case DUO_ETIMEOUT: return "a bounded device-side wait ran out";
+    default: return "unknown status code";
+  }
+}
+
+int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int fmt, void* stream,
+             duo_packed** h_out) {
+  if (W_fp16_dev == nullptr || h_out == nullptr) return DUO_EINVAL;
+  if (out < 1 || in < 1 || ldw < in) return DUO_EINVAL;
+  if (fmt != DUO_FMT_IDX16 && fmt != DUO_FMT_BITMASK) return DUO_EINVAL;
+  if (!aligned(W_fp16_dev, 2)) return DUO_EINVAL;
+  if (in > 65535) return DUO_ERANGE;
+  if (fmt == DUO_FMT_IDX16 && out > 65536) return DUO_ERANGE;
+  const int64_t S = (out + duo::kSegRows - 1) / duo::kSegRows;
+  if (S > 65535 || in * S + 1 > (int64_t)1 << 31) return DUO_ERANGE;
+  int rc = cuda_ready();
+  if (rc != DUO_OK) return rc;
+  if (!is_device_ptr(W_fp16_dev)) return DUO_EINVAL;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const uint16_t* W = static_cast<const uint16_t*>(W_fp16_dev);
+
+  Scratch scratch;
+  uint32_t* cnt_js = nullptr;
+  unsigned long long* totals = nullptr;
+  cudaError_t e = duo_malloc(reinterpret_cast<void**>(&cnt_js), sizeof(uint32_t) * in * S);
+  if (e != cudaSuccess) return map_err(e);
+  scratch.add(cnt_js);
+  e = duo_malloc(reinterpret_cast<void**>(&totals), 2 * sizeof(unsigned long long));
+  if (e != cudaSuccess) return map_err(e);
+  scratch.add(totals);
+
+  e = duo::launch_pack_count(W, out, in, ldw, (int)S, cnt_js, st);
+  if (e != cudaSuccess) return map_err(e);
+
+  duo_packed* h = new (std::nothrow) duo_packed();
+  if (h == nullptr) return DUO_ENOMEM;
+  h->fmt = fmt;
+  h->out = out;
+  h->in = in;
+  cudaGetDevice(&h->device);
+  void* index = nullptr;
+  void* aux = nullptr;
+  void* data = nullptr;
+  auto fail = [&](int code) {
+    if (index) cudaFree(index);
+    if (aux) cudaFree(aux);
+    if (data) cudaFree(data);
+    delete h;
+    return code;
+  };
+
+  unsigned long long host_tot[2] = {0, 0};
+  if (fmt == DUO_FMT_BITMASK) {
+    h->nseg = S;
+    h->index_bytes = (int64_t)sizeof(uint32_t) * (in * S + 1);
+    // The offsets are followed (at a 256-byte boundary) by the two barrier
+    // words of the spMspV kernel, zeroed here.
+    const size_t sync_at = (size_t)(h->index_bytes + 255) / 256 * 256;
+    e = duo_malloc(&index, sync_at + 256);
+    if (e != cudaSuccess) return fail(map_err(e));
+    h->sync = reinterpret_cast<unsigned int*>(static_cast<char*>(index) + sync_at);
+    e = cudaMemsetAsync(h->sync, 0, 256, st);
+    if (e != cudaSuccess) return fail(map_err(e));
+    e = duo::launch_cmb_offsets(cnt_js, in * S, static_cast<uint32_t*>(index), totals, st);
+    if (e != cudaSuccess) return fail(map_err(e));
+    e = cudaMemcpyAsync(host_tot, totals, sizeof(host_tot), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return fail(map_err(e));
+    if (host_tot[0] >= (1ull << 32)) return fail(DUO_ERANGE);
+    h->data_bytes = (int64_t)host_tot[0] * 16;
+    e = duo_malloc(&data, (size_t)h->data_bytes);
+    if (e != cudaSuccess) return fail(map_err(e));
+    e = cudaMemsetAsync(data, 0, (size_t)h->data_bytes, st);
+    if (e != cudaSuccess) return fail(map_err(e));
+    e = duo::launch_cmb_scatter(W, out, in, ldw, (int)S, static_cast<const uint32_t*>(index),
+                                static_cast<uint8_t*>(data), st);
+    if (e != cudaSuccess) return fail(map_err(e));
+  } else {
+    h->nseg = 0;
+    h->index_bytes = (int64_t)sizeof(uint64_t) * (in + 1);
+    h->aux_bytes = (int64_t)sizeof(uint32_t) * in;
+    e = duo_malloc(&index, (size_t)h->index_bytes);
+    if (e != cudaSuccess) return fail(map_err(e));
+    e = duo_malloc(&aux, (size_t)h->aux_bytes);
+    if (e != cudaSuccess) return fail(map_err(e));
+    e = duo::launch_idx16_offsets(cnt_js, in, (int)S, static_cast<uint32_t*>(aux),
+                                  static_cast<uint64_t*>(index), totals, st);
+    if (e != cudaSuccess) return fail(map_err(e));
+    e = cudaMemcpyAsync(host_tot, totals, sizeof(host_tot), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return fail(map_err(e));
+    h->data_bytes = (int64_t)host_tot[0];
+    e = duo_malloc(&data, (size_t)h->data_bytes);
+    if (e != cudaSuccess) return fail(map_err(e));
+    e = cudaMemsetAsync(data, 0, (size_t)h->data_bytes, st);
+    if (e != cudaSuccess) return fail(map_err(e));
+    e = duo::launch_idx16_scatter(W, out, in, ldw, (int)S, cnt_js, static_cast<const uint32_t*>(aux),
+                                  static_cast<const uint64_t*>(index), static_cast<uint8_t*>(data),
+                                  st);
+    if (e != cudaSuccess) return fail(map_err(e));
+  }
+  e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return fail(map_err(e));
+  h->nnz = (int64_t)host_tot[1];
+  h->index = index;
+  h->aux = aux;
+  h->data = data;
+  h->magic = kHandleMagic;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    live_handles().insert(h);
+  }
+  *h_out = h;
+  return DUO_OK;
+}
+
+int duo_sparsify(const void* x_fp16_dev, int64_t in, int64_t k, uint16_t* kept_idx_dev,
+                 void* kept_val_fp16_dev, void* stream) {
+  if (x_fp16_dev == nullptr) return DUO_EINVAL;
+  if (in < 1 || in > 65535 || k < 0 || k > in) return DUO_EINVAL;
+  if (k > 0 && (kept_idx_dev == nullptr || kept_val_fp16_dev == nullptr)) return DUO_EINVAL;
+  if (!aligned(x_fp16_dev, 2) || !aligned(kept_idx_dev, 2) || !aligned(kept_val_fp16_dev, 2))
+    return DUO_EINVAL;
+  int rc = cuda_ready();
+  if (rc != DUO_OK) return rc;
+  if (k == 0) return DUO_OK;
+  cudaError_t e = duo::launch_sparsify(static_cast<const uint16_t*>(x_fp16_dev), (int)in, (int)k,
+                                       kept_idx_dev, static_cast<uint16_t*>(kept_val_fp16_dev),
+                                       static_cast<cudaStream_t>(stream));
+  return map_err(e);
+}
+
+static int spmspv_common(const duo_packed* const* hs, int n, const void* x, const uint16_t* kidx,
+                         const void* kval, int64_t k, float* const* ys, void* stream) {
+  if (hs == nullptr || ys == nullptr || n < 1 || n > duo::kMaxProblems) return DUO_EINVAL;
+  const bool listed = kidx != nullptr || kval != nullptr;
+  if (listed && (kidx == nullptr || kval == nullptr)) return DUO_EINVAL;
+  if (!listed && x == nullptr) return DUO_EINVAL;
+  if (!aligned(x, 2) || !aligned(kidx, 2) || !aligned(kval, 2)) return DUO_EINVAL;
+  for (int p = 0; p < n; ++p) {
+    if (hs[p] == nullptr || ys[p] == nullptr) return DUO_EINVAL;
+    if (!aligned(ys[p], 16)) return DUO_EINVAL;
+    if (!is_live(hs[p])) return DUO_EINVAL;
+  }
+  const int64_t I = hs[0]->in;
+  for (int p = 1; p < n; ++p) {
+    if (hs[p]->in != I) return DUO_EINVAL;
+    if (hs[p]->fmt != DUO_FMT_BITMASK) return DUO_EFORMAT;
+  }
+  if (n > 1 && hs[0]->fmt != DUO_FMT_BITMASK) return DUO_EFORMAT;
+  if (k < 0 || k > I) return DUO_EINVAL;
+  int rc = cuda_ready();
+  if (rc != DUO_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (k == 0 || hs[0]->fmt != DUO_FMT_BITMASK) {
+    // The bitmask kernel zeroes y itself; other paths clear it here.
+    for (int p = 0; p < n; ++p) {
+      cudaError_t e = cudaMemsetAsync(ys[p], 0, sizeof(float) * (size_t)hs[p]->out, st);
+      if (e != cudaSuccess) return map_err(e);
+    }
+  }
+  if (k == 0) return DUO_OK;
+  cudaError_t e;
+  if (hs[0]->fmt == DUO_FMT_BITMASK) {
+    duo::CmbArgs a{};
+    a.np = n;
+    a.I = (int)I;
+    a.k = (int)k;
+    a.x = static_cast<const uint16_t*>(x);
+    a.kidx = listed ? kidx : nullptr;
+    a.kval = listed ? static_cast<const uint16_t*>(kval) : nullptr;
+    a.bar = hs[0]->sync;
+    for (int p = 0; p < n; ++p) {
+      a.p[p].data = static_cast<const uint8_t*>(hs[p]->data);
+      a.p[p].off = static_cast<const uint32_t*>(hs[p]->index);
+      a.p[p].y = ys[p];
+      a.p[p].O = (int)hs[p]->out;
+      a.p[p].S = (int)hs[p]->nseg;
+    }
+    e = duo::launch_cmb_spmspv(a, st);
+    if (e == cudaErrorInvalidValue) return DUO_ERANGE;
+  } else {
+    const duo_packed* h = hs[0];
+    duo::Idx16Args a{};
+    a.data = static_cast<const uint8_t*>(h->data);
+    a.colptr = static_cast<const uint64_t*>(h->index);
+    a.cnt = static_cast<const uint32_t*>(h->aux);
+    a.y = ys[0];
+    a.O = (int)h->out;
+    a.I = (int)I;
+    a.k = (int)k;
+    a.x = static_cast<const uint16_t*>(x);
+    a.kidx = listed ? kidx : nullptr;
+    a.kval = listed ? static_cast<const uint16_t*>(kval) : nullptr;
+    e = duo::launch_idx16_spmspv(a, st);
+  }
+  return map_err(e);
+}
+
+int duo_spmspv(const duo_packed* h, const void* x_fp16_dev, const uint16_t* kept_idx_dev,
+               const void* kept_val_fp16_dev, int64_t k, float* y_dev, void* stream) {
+  const duo_packed* hs[1] = {h};
+  float* ys[1] = {y_dev};
+  return spmspv_common(hs, 1, x_fp16_dev, kept_idx_dev, kept_val_fp16_dev, k, ys, stream);
+}
+
+int duo_spmspv_multi(const duo_packed* const* hs, int n, const void* x_fp16_dev,
+                     const uint16_t* kept_idx_dev, const void* kept_val_fp16_dev, int64_t k,
+                     float* const* ys_dev, void* stream) {
+  return spmspv_common(hs, n, x_fp16_dev, kept_idx_dev, kept_val_fp16_dev, k, ys_dev, stream);
+}
+
+int duo_free(duo_packed* h) {
+  if (h == nullptr) return DUO_OK;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto& s = live_handles();
+    auto it = s.find(h);
+    if (it == s.end()) return DUO_EINVAL;
+    s.erase(it);
+  }
+  h->magic = 0;
+  cudaError_t e1 = h->index ? cudaFree(h->index) : cudaSuccess;
+  cudaError_t e2 = h->aux ? cudaFree(h->aux) : cudaSuccess;
+  cudaError_t e3 = h->data ? cudaFree(h->data) : cudaSuccess;
+  delete h;
+  if (e1 != cudaSuccess) return map_err(e1);
+  if (e2 != cudaSuccess) return map_err(e2);
+  return map_err(e3);
+}
+
+int duo_packed_query(const duo_packed* h, duo_packed_info* info) {
+  if (h == nullptr || info == nullptr || !is_live(h)) return DUO_EINVAL;
+  std::memset(info, 0, sizeof(*info));
+  info->fmt = h->fmt;
+  info->version = h->fmt == DUO_FMT_BITMASK ? 1 : 0;
+  info->magic = h->fmt == DUO_FMT_BITMASK ? kCmbMagic : kIdx16Magic;
+  info->seg_rows = h->fmt == DUO_FMT_BITMASK ? duo::kSegRows : 0;
+  info->out = h->out;
+  info->in = h->in;
+  info->nseg = h->nseg;
+  info->nnz = h->nnz;
+  info->index_dev = h->index;
+  info->index_bytes = h->index_bytes;
+  info->aux_dev = h->aux;
+  info->aux_bytes = h->aux_bytes;
+  info->data_dev = h->data;
+  info->data_bytes = h->data_bytes;
+  return DUO_OK;
+}
+
+int duo_packed_export(const duo_packed* h, int which, void* dst_host, int64_t bytes) {
+  if (h == nullptr || dst_host == nullptr || !is_live(h)) return DUO_EINVAL;
+  const void* src = nullptr;
+  int64_t n = 0;
+  switch (which) {
+    case 0: src = h->index; n = h->index_bytes; break;
+    case 1: src = h->aux; n = h->aux_bytes; break;
+    case 2: src = h->data; n = h->data_bytes; break;
+    default: return DUO_EINVAL;
+  }
+  if (bytes != n) return DUO_EINVAL;
+  if (n == 0) return DUO_OK;
+  int rc = cuda_ready();
+  if (rc != DUO_OK) return rc;
+  return map_err(cudaMemcpy(dst_host, src, (size_t)n, cudaMemcpyDeviceToHost));
+}
+
+int duo_device_status(void* stream) {
+  int rc = cuda_ready();
+  if (rc != DUO_OK) return rc;
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return DUO_ECUDA;
+  unsigned int st = 0;
+  e = duo::read_and_clear_status(&st);
+  if (e != cudaSuccess) return DUO_ECUDA;
+  if (st & 1u) return DUO_ETIMEOUT;
+  if (st & 2u) return DUO_EFORMAT;
+  return DUO_OK;
+}
+
+}  // extern "C"

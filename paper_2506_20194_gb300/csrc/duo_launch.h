@@ -1,0 +1,79 @@
+// Host-side interface between the C ABI (api.cu) and the kernels
+// (kernels.cu).  Plain structs of device pointers and sizes.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace duo {
+
+constexpr int kMaxProblems = 4;
+constexpr int kSegRows = 1024;
+
+struct CmbProb {
+  const uint8_t* data;   // records
+  const uint32_t* off;   // off[I*S + 1], 16-byte units
+  float* y;              // fp32[O], zeroed before the launch
+  int O;
+  int S;
+};
+
+struct CmbArgs {
+  CmbProb p[kMaxProblems];
+  int np;
+  int I;
+  int k;
+  const uint16_t* x;     // fused mode: fp16 bits [I]
+  const uint16_t* kidx;  // listed mode: uint16 [k]
+  const uint16_t* kval;  // listed mode: fp16 bits [k]
+  unsigned int* bar;     // 2 words {count, generation} of a grid barrier, zero
+                         // between launches; owned by the first handle
+  int nslot;             // set by the launcher
+};
+
+struct Idx16Args {
+  const uint8_t* data;
+  const uint64_t* colptr;
+  const uint32_t* cnt;
+  float* y;
+  int O;
+  int I;
+  int k;
+  const uint16_t* x;
+  const uint16_t* kidx;
+  const uint16_t* kval;
+};
+
+// spMspV over the bitmask format (fused when a.kidx == nullptr).  Zeroes
+// every y itself (no memset needed before it).
+cudaError_t launch_cmb_spmspv(const CmbArgs& a, cudaStream_t st);
+// spMspV over the index format (fused when a.kidx == nullptr).
+cudaError_t launch_idx16_spmspv(const Idx16Args& a, cudaStream_t st);
+// Exact top-k sparsifier: kept ids ascending + their values.
+cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uint16_t* kval,
+                            cudaStream_t st);
+
+// Packing.  cnt_js[j*S + s] = non-zeros of channel j in row segment s.
+cudaError_t launch_pack_count(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
+                              uint32_t* cnt_js, cudaStream_t st);
+// off[n] exclusive prefix (16-byte units) of the CMB record sizes;
+// totals[0] = total units (64-bit), totals[1] = total non-zeros.
+cudaError_t launch_cmb_offsets(const uint32_t* cnt_js, int64_t n, uint32_t* off,
+                               unsigned long long* totals, cudaStream_t st);
+cudaError_t launch_cmb_scatter(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
+                               const uint32_t* off, uint8_t* data, cudaStream_t st);
+// cnt[j] = sum_s cnt_js, colptr[j] byte offsets of the IDX16 blocks;
+// totals[0] = total bytes, totals[1] = total non-zeros.
+cudaError_t launch_idx16_offsets(const uint32_t* cnt_js, int64_t I, int S, uint32_t* cnt,
+                                 uint64_t* colptr, unsigned long long* totals, cudaStream_t st);
+cudaError_t launch_idx16_scatter(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
+                                 const uint32_t* cnt_js, const uint32_t* cnt,
+                                 const uint64_t* colptr, uint8_t* data, cudaStream_t st);
+
+// Reads and clears the device status word (bit 0: a bounded wait ran out,
+// bit 1: a record size outside the format's bounds).
+cudaError_t read_and_clear_status(unsigned int* out);
+
+}  // namespace duo

@@ -1,0 +1,718 @@
+// Kernels of libduo (sm_103a): the channel-major packer (§4.1 storage), the
+// exact magnitude top-k sparsifier (§3), and the dual-sparse spMspV
+// y = W (x ⊙ m^x) (§3) over the bitmask ("CMB") and index ("IDX16")
+// formats.  All device code lives in this one translation unit so the
+// device status word needs no relocatable device code.
+#include <algorithm>
+#include <cstdio>
+
+#include "duo_device.cuh"
+#include "duo_launch.h"
+
+namespace duo {
+
+// ------------------------------------------------------------------------
+// Device properties (cached per device).
+// ------------------------------------------------------------------------
+struct DevProps {
+  int nsm = 0;
+  int smem_optin = 0;
+};
+
+static cudaError_t dev_props(DevProps* out) {
+  static DevProps cache[64];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (cache[dev].nsm == 0) {
+    DevProps p;
+    e = cudaDeviceGetAttribute(&p.nsm, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&p.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e != cudaSuccess) return e;
+    cache[dev] = p;
+  }
+  *out = cache[dev];
+  return cudaSuccess;
+}
+
+__host__ __device__ inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// ------------------------------------------------------------------------
+// Packing (§4.1: each kept column is stored compressed; column-major
+// storage per the footnote of §3).  A CTA loads a 1024-row x 32-channel tile
+// of the row-major weight with coalesced loads into shared memory (row pitch
+// 34 halves so that the column walk below is bank-conflict free); warp w
+// then walks channels w, w+8, ...: for mask word t, lane b tests row 32t+b,
+// a ballot gives the word, and popcounts give each value's slot.
+// ------------------------------------------------------------------------
+constexpr int PACK_THREADS = 256;
+constexpr int PACK_PITCH = 34;  // halves per tile row
+constexpr size_t PACK_SMEM = (size_t)SEG_ROWS * PACK_PITCH * 2;
+
+enum PackMode { PACK_COUNT = 0, PACK_CMB = 1, PACK_IDX16 = 2 };
+
+struct PackArgs {
+  const uint16_t* W;
+  int64_t O, I, ldw;
+  int S;
+  uint32_t* cnt_js;          // COUNT: output
+  const uint32_t* cnt_js_in; // IDX16: per-segment counts
+  const uint32_t* off;       // CMB
+  const uint32_t* cnt;       // IDX16
+  const uint64_t* colptr;    // IDX16
+  uint8_t* data;
+};
+
+template <int MODE>
+__global__ void __launch_bounds__(PACK_THREADS) pack_tile_kernel(const PackArgs a) {
+  extern __shared__ __align__(16) uint16_t tile[];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t j0 = (int64_t)blockIdx.x * 32;
+  const int s = blockIdx.y;
+  const int64_t r0 = (int64_t)s * SEG_ROWS;
+  const int64_t rows64 = a.O - r0;
+  const int rows = rows64 < SEG_ROWS ? (int)rows64 : SEG_ROWS;
+  const int64_t ncol64 = a.I - j0;
+  const int ncol = ncol64 < 32 ? (int)ncol64 : 32;
+  for (int e = tid; e < SEG_ROWS * 32; e += PACK_THREADS) {
+    const int r = e >> 5, c = e & 31;
+    uint16_t v = 0;
+    if (r < rows && c < ncol) v = a.W[(r0 + r) * a.ldw + j0 + c];
+    tile[r * PACK_PITCH + c] = v;
+  }
+  __syncthreads();
+  const uint32_t lt = (1u << lane) - 1u;
+  for (int c = warp; c < ncol; c += PACK_THREADS / 32) {
+    const int64_t j = j0 + c;
+    uint32_t total = 0, myword = 0;
+    uint16_t* vals = nullptr;
+    uint16_t* rowids = nullptr;
+    if (MODE == PACK_CMB) {
+      const uint32_t o = a.off[j * a.S + s];
+      vals = reinterpret_cast<uint16_t*>(a.data + (size_t)o * 16 + MASK_BYTES);
+    } else if (MODE == PACK_IDX16) {
+      uint32_t pre = 0;
+      for (int s2 = 0; s2 < s; ++s2) pre += a.cnt_js_in[j * a.S + s2];
+      const uint32_t n = a.cnt[j];
+      uint8_t* blk = a.data + a.colptr[j];
+      vals = reinterpret_cast<uint16_t*>(blk) + pre;
+      rowids = reinterpret_cast<uint16_t*>(blk + align_up((size_t)2 * n, 16)) + pre;
+    }
+#pragma unroll 4
+    for (int t = 0; t < SEG_WORDS; ++t) {
+      const uint16_t v = tile[(32 * t + lane) * PACK_PITCH + c];
+      const bool nz = (v & 0x7FFFu) != 0u;
+      const uint32_t word = __ballot_sync(FULL_MASK, nz);
+      if (MODE == PACK_CMB) {
+        if (lane == t) myword = word;
+        if (nz) vals[total + __popc(word & lt)] = v;
+      } else if (MODE == PACK_IDX16) {
+        if (nz) {
+          const uint32_t pos = total + __popc(word & lt);
+          vals[pos] = v;
+          rowids[pos] = (uint16_t)(r0 + 32 * t + lane);
+        }
+      }
+      total += __popc(word);
+    }
+    if (MODE == PACK_COUNT) {
+      if (lane == 0) a.cnt_js[j * a.S + s] = total;
+    } else if (MODE == PACK_CMB) {
+      const uint32_t o = a.off[j * a.S + s];
+      reinterpret_cast<uint32_t*>(a.data + (size_t)o * 16)[lane] = myword;
+    }
+  }
+}
+
+static cudaError_t launch_pack_tiles(int mode, const PackArgs& a, cudaStream_t st) {
+  const dim3 grid((unsigned)((a.I + 31) / 32), (unsigned)a.S);
+  cudaError_t e;
+  switch (mode) {
+    case PACK_COUNT:
+      e = cudaFuncSetAttribute(pack_tile_kernel<PACK_COUNT>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PACK_SMEM);
+      if (e != cudaSuccess) return e;
+      pack_tile_kernel<PACK_COUNT><<<grid, PACK_THREADS, PACK_SMEM, st>>>(a);
+      break;
+    case PACK_CMB:
+      e = cudaFuncSetAttribute(pack_tile_kernel<PACK_CMB>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PACK_SMEM);
+      if (e != cudaSuccess) return e;
+      pack_tile_kernel<PACK_CMB><<<grid, PACK_THREADS, PACK_SMEM, st>>>(a);
+      break;
+    default:
+      e = cudaFuncSetAttribute(pack_tile_kernel<PACK_IDX16>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PACK_SMEM);
+      if (e != cudaSuccess) return e;
+      pack_tile_kernel<PACK_IDX16><<<grid, PACK_THREADS, PACK_SMEM, st>>>(a);
+      break;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pack_count(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
+                              uint32_t* cnt_js, cudaStream_t st) {
+  PackArgs a{};
+  a.W = W; a.O = O; a.I = I; a.ldw = ldw; a.S = S; a.cnt_js = cnt_js;
+  return launch_pack_tiles(PACK_COUNT, a, st);
+}
+
+cudaError_t launch_cmb_scatter(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
+                               const uint32_t* off, uint8_t* data, cudaStream_t st) {
+  PackArgs a{};
+  a.W = W; a.O = O; a.I = I; a.ldw = ldw; a.S = S; a.off = off; a.data = data;
+  return launch_pack_tiles(PACK_CMB, a, st);
+}
+
+cudaError_t launch_idx16_scatter(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
+                                 const uint32_t* cnt_js, const uint32_t* cnt,
+                                 const uint64_t* colptr, uint8_t* data, cudaStream_t st) {
+  PackArgs a{};
+  a.W = W; a.O = O; a.I = I; a.ldw = ldw; a.S = S; a.cnt_js_in = cnt_js; a.cnt = cnt;
+  a.colptr = colptr; a.data = data;
+  return launch_pack_tiles(PACK_IDX16, a, st);
+}
+
+// Single-CTA chunked exclusive scan (packing is an offline step; one CTA
+// walking a few million entries takes well under a millisecond).
+constexpr int SCAN_THREADS = 1024;
+constexpr int SCAN_PER = 8;
+
+template <typename F, typename G>
+__device__ void chunked_scan(int64_t n, F value, G emit, unsigned long long* total_out) {
+  __shared__ unsigned long long wsum[32];
+  __shared__ unsigned long long carry;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  if (tid == 0) carry = 0ull;
+  __syncthreads();
+  for (int64_t base = 0; base < n; base += (int64_t)SCAN_THREADS * SCAN_PER) {
+    unsigned long long v[SCAN_PER], s = 0;
+#pragma unroll
+    for (int q = 0; q < SCAN_PER; ++q) {
+      const int64_t i = base + (int64_t)tid * SCAN_PER + q;
+      v[q] = i < n ? value(i) : 0ull;
+      s += v[q];
+    }
+    unsigned long long inc = s;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned long long t = __shfl_up_sync(FULL_MASK, inc, o);
+      if (lane >= o) inc += t;
+    }
+    if (lane == 31) wsum[wid] = inc;
+    __syncthreads();
+    if (wid == 0) {
+      unsigned long long w = wsum[lane];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long t = __shfl_up_sync(FULL_MASK, w, o);
+        if (lane >= o) w += t;
+      }
+      wsum[lane] = w;
+    }
+    __syncthreads();
+    unsigned long long run = carry + (wid > 0 ? wsum[wid - 1] : 0ull) + inc - s;
+#pragma unroll
+    for (int q = 0; q < SCAN_PER; ++q) {
+      const int64_t i = base + (int64_t)tid * SCAN_PER + q;
+      if (i < n) emit(i, run);
+      run += v[q];
+    }
+    __syncthreads();
+    if (tid == 0) carry += wsum[31];
+    __syncthreads();
+  }
+  if (tid == 0) *total_out = carry;
+}
+
+__global__ void __launch_bounds__(SCAN_THREADS) cmb_offsets_kernel(const uint32_t* cnt_js, int64_t n,
+                                                                   uint32_t* off,
+                                                                   unsigned long long* totals) {
+  // record units = (128 + pad16(2 * cnt)) / 16 = 8 + ceil(cnt / 8)
+  chunked_scan(
+      n, [&](int64_t i) { return 8ull + (cnt_js[i] + 7ull) / 8ull; },
+      [&](int64_t i, unsigned long long pre) { off[i] = (uint32_t)pre; }, &totals[0]);
+  __syncthreads();
+  chunked_scan(
+      n, [&](int64_t i) { return (unsigned long long)cnt_js[i]; },
+      [&](int64_t, unsigned long long) {}, &totals[1]);
+  __syncthreads();
+  if (threadIdx.x == 0) off[n] = (uint32_t)totals[0];
+}
+
+cudaError_t launch_cmb_offsets(const uint32_t* cnt_js, int64_t n, uint32_t* off,
+                               unsigned long long* totals, cudaStream_t st) {
+  cmb_offsets_kernel<<<1, SCAN_THREADS, 0, st>>>(cnt_js, n, off, totals);
+  return cudaGetLastError();
+}
+
+__global__ void __launch_bounds__(SCAN_THREADS) idx16_offsets_kernel(const uint32_t* cnt_js,
+                                                                     int64_t I, int S,
+                                                                     uint32_t* cnt,
+                                                                     uint64_t* colptr,
+                                                                     unsigned long long* totals) {
+  for (int64_t j = threadIdx.x; j < I; j += SCAN_THREADS) {
+    uint32_t c = 0;
+    for (int s = 0; s < S; ++s) c += cnt_js[j * S + s];
+    cnt[j] = c;
+  }
+  __syncthreads();
+  chunked_scan(
+      I, [&](int64_t j) { return 2ull * align_up(2ull * cnt[j], 16ull); },
+      [&](int64_t j, unsigned long long pre) { colptr[j] = pre; }, &totals[0]);
+  __syncthreads();
+  chunked_scan(
+      I, [&](int64_t j) { return (unsigned long long)cnt[j]; },
+      [&](int64_t, unsigned long long) {}, &totals[1]);
+  __syncthreads();
+  if (threadIdx.x == 0) colptr[I] = totals[0];
+}
+
+cudaError_t launch_idx16_offsets(const uint32_t* cnt_js, int64_t I, int S, uint32_t* cnt,
+                                 uint64_t* colptr, unsigned long long* totals, cudaStream_t st) {
+  idx16_offsets_kernel<<<1, SCAN_THREADS, 0, st>>>(cnt_js, I, S, cnt, colptr, totals);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------------
+// Sparsifier (§3): one CTA selects and compacts the kept channels.
+// ------------------------------------------------------------------------
+constexpr int SPARSIFY_THREADS = 1024;
+
+struct SelLayout {
+  size_t xs, kb, kp, eqw, sel, end;
+};
+
+__host__ __device__ inline SelLayout sel_layout(int I, size_t base) {
+  const size_t nw = (size_t)(I + 31) / 32;
+  SelLayout L;
+  size_t o = base;
+  L.xs = o;  o += align_up(2 * (size_t)I, 16);
+  L.kb = o;  o += align_up(4 * nw, 16);
+  L.kp = o;  o += align_up(4 * (nw + 1), 16);
+  L.eqw = o; o += align_up(4 * nw, 16);
+  L.sel = o; o += align_up(sizeof(SelShared), 16);
+  L.end = o;
+  return L;
+}
+
+__global__ void __launch_bounds__(SPARSIFY_THREADS) sparsify_kernel(const uint16_t* __restrict__ x,
+                                                                    int I, int k,
+                                                                    uint16_t* __restrict__ kidx,
+                                                                    uint16_t* __restrict__ kval) {
+  extern __shared__ __align__(128) uint8_t sm[];
+  const SelLayout L = sel_layout(I, 0);
+  uint16_t* xs = reinterpret_cast<uint16_t*>(sm + L.xs);
+  uint32_t* kb = reinterpret_cast<uint32_t*>(sm + L.kb);
+  uint32_t* kp = reinterpret_cast<uint32_t*>(sm + L.kp);
+  uint32_t* eqw = reinterpret_cast<uint32_t*>(sm + L.eqw);
+  SelShared* sel = reinterpret_cast<SelShared*>(sm + L.sel);
+  load_x_to_smem(xs, x, I);
+  __syncthreads();
+  select_topk(xs, I, k, kb, kp, eqw, sel);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = (I + 31) >> 5;
+  for (int w = warp; w < nw; w += SPARSIFY_THREADS / 32) {
+    const uint32_t bits = kb[w];
+    if ((bits >> lane) & 1u) {
+      const uint32_t pos = kp[w] + __popc(bits & ((1u << lane) - 1u));
+      const int j = 32 * w + lane;
+      kidx[pos] = (uint16_t)j;
+      kval[pos] = xs[j];
+    }
+  }
+}
+
+cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uint16_t* kval,
+                            cudaStream_t st) {
+  const size_t smem = sel_layout(I, 0).end;
+  cudaError_t e = cudaFuncSetAttribute(sparsify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  sparsify_kernel<<<1, SPARSIFY_THREADS, smem, st>>>(x, I, k, kidx, kval);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------------
+// spMspV over the bitmask format (§3 product, §4.1 "only the rows ... of
+// non-zero activations are fetched").
+//
+// Persistent CTAs, one per SM.  The work items are (product p, row segment
+// s, kept index i), ordered p, s, i; CTA b takes the contiguous item range
+// [total*b/G, total*(b+1)/G).  Warp 0 is the producer: its 32 lanes each
+// resolve one item (kept channel id, record offset and size) and issue a
+// 1-D bulk copy of the record into a ring slot in shared memory, signalled
+// on the slot's "full" mbarrier.  Warps 1..NC consume: item v goes to
+// consumer v % NC and slot v % nslot.  A consumer owns, for the current
+// segment, rows 32*lane .. 32*lane+31 in 32 fp32 registers: it reads its
+// mask word, finds where its values start with a warp prefix sum of
+// popcounts, and walks its bits, multiplying each stored fp16 weight by the
+// channel's fp16 activation with an fp32 accumulation.  When a segment ends
+// the consumers add their registers into a shared-memory row tile (rotated
+// so that lanes hit distinct banks) and add the tile to y with vector
+// reductions.
+//
+// y is zeroed by the kernel itself: each CTA clears a slice of the outputs
+// at the start and arrives on a split-phase grid barrier; a CTA waits on it
+// only before its first reduction into y, by which time every CTA has long
+// arrived.  The launch is cooperative, so all CTAs are co-resident.
+// ------------------------------------------------------------------------
+constexpr int CMB_NC = 16;
+constexpr int CMB_THREADS = 32 * (1 + CMB_NC);
+constexpr int CMB_MAX_SLOTS = 64;
+
+struct CmbLayout {
+  SelLayout sel;
+  size_t tile, full, empty, meta, ring, total;
+};
+
+__host__ __device__ inline CmbLayout cmb_layout(int I, bool fused, int nslot) {
+  CmbLayout L;
+  size_t o = 0;
+  if (fused) {
+    L.sel = sel_layout(I, 0);
+    o = L.sel.end;
+  }
+  L.tile = o;  o += 2 * SEG_ROWS * sizeof(float);
+  L.full = o;  o += 8 * (size_t)nslot;
+  L.empty = o; o += 8 * (size_t)nslot;
+  L.meta = o;  o += align_up(4 * (size_t)nslot, 16);
+  o = align_up(o, 128);
+  L.ring = o;  o += (size_t)nslot * MAX_RECORD_BYTES;
+  L.total = o;
+  return L;
+}
+
+__device__ __forceinline__ int tile_index(int r) { return (r & ~31) | ((r + (r >> 5)) & 31); }
+
+// One consumer warp decodes one record: lane owns rows 32*lane + t.
+__device__ __forceinline__ void decode_record(const uint8_t* rec, uint16_t xb, float (&acc)[32],
+                                              int lane) {
+  const uint32_t m = reinterpret_cast<const uint32_t*>(rec)[lane];
+  const uint32_t c = __popc(m);
+  const uint32_t incl = warp_inclusive_scan(c, lane);
+  const uint16_t* vp = reinterpret_cast<const uint16_t*>(rec + MASK_BYTES) + (incl - c);
+#pragma unroll
+  for (int t = 0; t < 32; ++t) {
+    if (m & (1u << t)) {
+      acc[t] = fma_f16_f32(*vp, xb, acc[t]);
+      ++vp;
+    }
+  }
+}
+
+// Decodes work item u into (product p, segment s, kept index i).
+__device__ __forceinline__ void cmb_item(const CmbArgs& a, int64_t u, int& p, int& s, int& i,
+                                         int64_t& seg_end) {
+  const int64_t k = a.k;
+  int64_t base = 0;
+  p = 0;
+  while (p < a.np - 1 && u >= base + (int64_t)a.p[p].S * k) {
+    base += (int64_t)a.p[p].S * k;
+    ++p;
+  }
+  const int64_t rem = u - base;
+  s = (int)(rem / k);
+  i = (int)(rem - (int64_t)s * k);
+  seg_end = base + (int64_t)(s + 1) * k;
+}
+
+template <bool FUSED>
+__global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArgs a) {
+  extern __shared__ __align__(128) uint8_t sm[];
+  __shared__ volatile int abort_flag;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nslot = a.nslot;
+  const CmbLayout L = cmb_layout(a.I, FUSED, nslot);
+  float* tile = reinterpret_cast<float*>(sm + L.tile);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sm + L.full);
+  uint64_t* empty = reinterpret_cast<uint64_t*>(sm + L.empty);
+  uint32_t* meta = reinterpret_cast<uint32_t*>(sm + L.meta);
+  uint8_t* ring = sm + L.ring;
+  uint16_t* xs = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.xs) : nullptr;
+  uint32_t* kb = FUSED ? reinterpret_cast<uint32_t*>(sm + L.sel.kb) : nullptr;
+  uint32_t* kp = FUSED ? reinterpret_cast<uint32_t*>(sm + L.sel.kp) : nullptr;
+  const int nw = (a.I + 31) >> 5;
+
+  if (tid == 0) abort_flag = 0;
+  for (int i = tid; i < nslot; i += CMB_THREADS) {
+    mbar_init(&full[i], 1);
+    mbar_init(&empty[i], 1);
+  }
+  for (int i = tid; i < 2 * SEG_ROWS; i += CMB_THREADS) tile[i] = 0.f;
+  if (FUSED) load_x_to_smem(xs, a.x, a.I);
+  fence_mbar_init();
+  __syncthreads();
+  // Zero this CTA's slice of the outputs, then arrive on the grid barrier.
+  {
+    int64_t ytot = 0;
+    for (int p = 0; p < a.np; ++p) ytot += a.p[p].O;
+    const int64_t z0 = ytot * blockIdx.x / gridDim.x, z1 = ytot * (blockIdx.x + 1) / gridDim.x;
+    int64_t base = 0;
+    for (int p = 0; p < a.np; ++p) {
+      const int64_t lo = z0 > base ? z0 : base;
+      const int64_t hi = z1 < base + a.p[p].O ? z1 : base + a.p[p].O;
+      for (int64_t r = lo + tid; r < hi; r += CMB_THREADS) a.p[p].y[r - base] = 0.f;
+      base += a.p[p].O;
+    }
+  }
+  if (FUSED) {
+    select_topk(xs, a.I, a.k, kb, kp, reinterpret_cast<uint32_t*>(sm + L.sel.eqw),
+                reinterpret_cast<SelShared*>(sm + L.sel.sel));
+  } else {
+    __syncthreads();
+  }
+  __shared__ unsigned int bar_gen0;
+  if (tid == 0) {
+    __threadfence();
+    bar_gen0 = ld_acquire_gpu(a.bar + 1);
+    if (atomicAdd(a.bar, 1u) == gridDim.x - 1) {
+      a.bar[0] = 0u;
+      __threadfence();
+      atomicAdd(a.bar + 1, 1u);
+    }
+  }
+  __syncthreads();   // publishes bar_gen0
+
+  const int64_t k = a.k;
+  int64_t total = 0;
+  for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * k;
+  const int64_t u0 = total * blockIdx.x / gridDim.x;
+  const int64_t u1 = total * (blockIdx.x + 1) / gridDim.x;
+  const int64_t nv = u1 - u0;
+
+  if (warp == 0) {
+    // ---------------- producer ----------------
+    const uint64_t pol = policy_evict_first();
+    int64_t last_v = -1;
+    for (int64_t vb = 0; vb < nv; vb += 32) {
+      if (abort_flag) break;
+      const int64_t v = vb + lane;
+      if (v >= nv) continue;
+      int p, s, i;
+      int64_t seg_end;
+      cmb_item(a, u0 + v, p, s, i, seg_end);
+      int j;
+      uint16_t xb;
+      if (FUSED) {
+        j = kept_channel(kb, kp, nw, (uint32_t)i);
+        xb = xs[j];
+      } else {
+        j = __ldg(a.kidx + i);
+        xb = __ldg(a.kval + i);
+      }
+      if (j < 0 || j >= a.I) {
+        atomicOr(&g_status, STATUS_FORMAT);
+        abort_flag = 1;
+        break;
+      }
+      const CmbProb& P = a.p[p];
+      const int64_t ri = (int64_t)j * P.S + s;
+      const uint32_t o0 = __ldg(P.off + ri), o1 = __ldg(P.off + ri + 1);
+      const uint32_t bytes = (o1 - o0) * 16u;
+      if (o1 < o0 || bytes < (uint32_t)MASK_BYTES || bytes > (uint32_t)MAX_RECORD_BYTES) {
+        atomicOr(&g_status, STATUS_FORMAT);
+        abort_flag = 1;
+        break;
+      }
+      const int slot = (int)(v % nslot);
+      const int64_t n = v / nslot;
+      if (n > 0 && !mbar_wait_bounded(&empty[slot], (uint32_t)((n - 1) & 1), &abort_flag)) break;
+      meta[slot] = xb;
+      mbar_arrive_expect_tx(&full[slot], bytes);
+      bulk_g2s(ring + (size_t)slot * MAX_RECORD_BYTES, P.data + (size_t)o0 * 16, bytes, &full[slot],
+               pol);
+      last_v = v;
+    }
+    if (abort_flag) {
+      // Let this lane's copies still in flight land before the CTA exits.
+      for (int64_t v = last_v; v >= 0 && v > last_v - nslot; v -= 32)
+        mbar_wait_limited(&full[v % nslot], (uint32_t)((v / nslot) & 1));
+    }
+  } else {
+    // ---------------- consumers ----------------
+    const int c = warp - 1;
+    const int ctid = tid - 32;
+    float acc[32];
+    int64_t u = u0;
+    int piece = 0;
+    while (u < u1) {
+      int p, s, i0;
+      int64_t seg_end;
+      cmb_item(a, u, p, s, i0, seg_end);
+      const int64_t pend = seg_end < u1 ? seg_end : u1;
+      const int64_t va = u - u0, vb = pend - u0;
+#pragma unroll
+      for (int t = 0; t < 32; ++t) acc[t] = 0.f;
+      bool any = false;
+      int64_t v = va + ((c - (int)(va % CMB_NC)) % CMB_NC + CMB_NC) % CMB_NC;
+      for (; v < vb; v += CMB_NC) {
+        const int slot = (int)(v % nslot);
+        const uint32_t par = (uint32_t)((v / nslot) & 1);
+        if (!abort_flag && mbar_wait_bounded(&full[slot], par, &abort_flag)) {
+          decode_record(ring + (size_t)slot * MAX_RECORD_BYTES, (uint16_t)meta[slot], acc, lane);
+          any = true;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[slot]);
+      }
+      float* tb = tile + (piece & 1) * SEG_ROWS;
+      if (any) {
+#pragma unroll
+        for (int t = 0; t < 32; ++t) atomicAdd(&tb[32 * lane + ((t + lane) & 31)], acc[t]);
+      }
+      if (piece == 0 && ctid == 0) {
+        // First reduction into y: every CTA must have zeroed its slice.
+        const uint64_t t0 = globaltimer_ns();
+        while (ld_acquire_gpu(a.bar + 1) == bar_gen0) {
+          if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
+            atomicOr(&g_status, STATUS_TIMEOUT);
+            abort_flag = 1;
+            break;
+          }
+        }
+      }
+      named_bar_sync(1, CMB_NC * 32);
+      const CmbProb& P = a.p[p];
+      const int rows = min(SEG_ROWS, P.O - s * SEG_ROWS);
+      float* yb = P.y + (size_t)s * SEG_ROWS;
+      for (int g = ctid; 4 * g < rows; g += CMB_NC * 32) {
+        float vv[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int r = 4 * g + e;
+          if (r < rows) {
+            const int ix = tile_index(r);
+            vv[e] = tb[ix];
+            tb[ix] = 0.f;
+          } else {
+            vv[e] = 0.f;
+          }
+        }
+        if (4 * g + 3 < rows) {
+          red_add_v4(yb + 4 * g, vv[0], vv[1], vv[2], vv[3]);
+        } else {
+          for (int e = 0; e < 4 && 4 * g + e < rows; ++e) atomicAdd(yb + 4 * g + e, vv[e]);
+        }
+      }
+      ++piece;
+      u = pend;
+    }
+  }
+}
+
+cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
+  CmbArgs a = a0;
+  DevProps dp;
+  cudaError_t e = dev_props(&dp);
+  if (e != cudaSuccess) return e;
+  const bool fused = a.kidx == nullptr;
+  const size_t fixed = cmb_layout(a.I, fused, 0).total + 256;
+  const size_t per_slot = MAX_RECORD_BYTES + 8 + 8 + 4;
+  int nslot = 0;
+  if ((size_t)dp.smem_optin > fixed) nslot = (int)(((size_t)dp.smem_optin - fixed) / per_slot);
+  nslot = std::min(nslot, CMB_MAX_SLOTS) / CMB_NC * CMB_NC;
+  if (nslot < 32) return cudaErrorInvalidValue;
+  a.nslot = nslot;
+  const size_t smem = cmb_layout(a.I, fused, nslot).total;
+  int64_t total = 0;
+  for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
+  if (total <= 0) return cudaSuccess;
+  const int grid = (int)std::min<int64_t>(dp.nsm, total);
+  void (*kern)(const CmbArgs) = fused ? cmb_spmspv_kernel<true> : cmb_spmspv_kernel<false>;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(CMB_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, a);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------------
+// spMspV over the index format (parity format): one warp per kept channel,
+// lanes stride its non-zeros and add w * x into y[row] atomically.
+// ------------------------------------------------------------------------
+constexpr int IDX16_THREADS = 256;
+
+template <bool FUSED>
+__global__ void __launch_bounds__(IDX16_THREADS) idx16_spmspv_kernel(const Idx16Args a) {
+  extern __shared__ __align__(128) uint8_t sm[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = (a.I + 31) >> 5;
+  const SelLayout L = sel_layout(a.I, 0);
+  uint16_t* xs = reinterpret_cast<uint16_t*>(sm + L.xs);
+  uint32_t* kb = reinterpret_cast<uint32_t*>(sm + L.kb);
+  uint32_t* kp = reinterpret_cast<uint32_t*>(sm + L.kp);
+  if (FUSED) {
+    load_x_to_smem(xs, a.x, a.I);
+    __syncthreads();
+    select_topk(xs, a.I, a.k, kb, kp, reinterpret_cast<uint32_t*>(sm + L.eqw),
+                reinterpret_cast<SelShared*>(sm + L.sel));
+  }
+  const int nwt = gridDim.x * (IDX16_THREADS / 32);
+  for (int i = blockIdx.x * (IDX16_THREADS / 32) + warp; i < a.k; i += nwt) {
+    int j;
+    uint16_t xb;
+    if (FUSED) {
+      j = kept_channel(kb, kp, nw, (uint32_t)i);
+      xb = xs[j];
+    } else {
+      j = __ldg(a.kidx + i);
+      xb = __ldg(a.kval + i);
+    }
+    if (j >= a.I) {
+      if (lane == 0) atomicOr(&g_status, STATUS_FORMAT);
+      continue;
+    }
+    const uint32_t n = __ldg(a.cnt + j);
+    const uint8_t* blk = a.data + __ldg(a.colptr + j);
+    const uint16_t* vals = reinterpret_cast<const uint16_t*>(blk);
+    const uint16_t* rows = reinterpret_cast<const uint16_t*>(blk + align_up((size_t)2 * n, 16));
+    for (uint32_t e = lane; e < n; e += 32) {
+      const uint32_t r = __ldg(rows + e);
+      if (r < (uint32_t)a.O) atomicAdd(a.y + r, fma_f16_f32(__ldg(vals + e), xb, 0.f));
+    }
+  }
+}
+
+cudaError_t launch_idx16_spmspv(const Idx16Args& a, cudaStream_t st) {
+  DevProps dp;
+  cudaError_t e = dev_props(&dp);
+  if (e != cudaSuccess) return e;
+  if (a.k <= 0) return cudaSuccess;
+  const bool fused = a.kidx == nullptr;
+  const size_t smem = fused ? sel_layout(a.I, 0).end : 0;
+  const int warps = IDX16_THREADS / 32;
+  const int grid = (int)std::min<int64_t>((int64_t)dp.nsm * 2, ((int64_t)a.k + warps - 1) / warps);
+  if (fused) {
+    e = cudaFuncSetAttribute(idx16_spmspv_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return e;
+    idx16_spmspv_kernel<true><<<grid, IDX16_THREADS, smem, st>>>(a);
+  } else {
+    idx16_spmspv_kernel<false><<<grid, IDX16_THREADS, 0, st>>>(a);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t read_and_clear_status(unsigned int* out) {
+  unsigned int v = 0, zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(&v, g_status, sizeof(v));
+  if (e != cudaSuccess) return e;
+  e = cudaMemcpyToSymbol(g_status, &zero, sizeof(zero));
+  *out = v;
+  return e;
+}
+
+}  // namespace duo

@@ -1,0 +1,209 @@
+"""Thin ctypes binding of libduo (include/duo.h): argument marshalling only.
+
+Every step of the compute path runs in the library's CUDA kernels; PyTorch
+only provides device memory and streams.  There is no fallback: if
+``libduo.so`` is missing or cannot be loaded, :func:`load_library` raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libduo.so")
+
+DUO_OK, DUO_EINVAL, DUO_ENOMEM, DUO_ECUDA, DUO_ERANGE, DUO_EFORMAT, DUO_ETIMEOUT = 0, -1, -2, -3, -4, -5, -6
+DUO_FMT_IDX16, DUO_FMT_BITMASK = 0, 1
+FORMATS = {"idx16": DUO_FMT_IDX16, "bitmask": DUO_FMT_BITMASK, "cmb": DUO_FMT_BITMASK}
+
+_lib = None
+
+
+class DuoError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        self.code = code
+        super().__init__(f"{what}: {duo_strerror(code)} ({code})")
+
+
+class _Info(ctypes.Structure):
+    _fields_ = [("fmt", ctypes.c_int32), ("version", ctypes.c_int32), ("magic", ctypes.c_uint32),
+                ("seg_rows", ctypes.c_int32), ("out", ctypes.c_int64), ("inp", ctypes.c_int64),
+                ("nseg", ctypes.c_int64), ("nnz", ctypes.c_int64),
+                ("index_dev", ctypes.c_void_p), ("index_bytes", ctypes.c_int64),
+                ("aux_dev", ctypes.c_void_p), ("aux_bytes", ctypes.c_int64),
+                ("data_dev", ctypes.c_void_p), ("data_bytes", ctypes.c_int64)]
+
+
+def load_library(path: str | None = None):
+    """Loads libduo.so (once).  Raises if it is missing: there is no
+    CPU or PyTorch fallback for any entry point."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"libduo.so not built ({p}); run paper_2506_20194_gb300.build")
+    lib = ctypes.CDLL(p)
+    vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+    lib.duo_pack.argtypes = [vp, i64, i64, i64, i32, vp, ctypes.POINTER(vp)]
+    lib.duo_sparsify.argtypes = [vp, i64, i64, vp, vp, vp]
+    lib.duo_spmspv.argtypes = [vp, vp, vp, vp, i64, vp, vp]
+    lib.duo_spmspv_multi.argtypes = [ctypes.POINTER(vp), i32, vp, vp, vp, i64, ctypes.POINTER(vp), vp]
+    lib.duo_free.argtypes = [vp]
+    lib.duo_packed_query.argtypes = [vp, ctypes.POINTER(_Info)]
+    lib.duo_packed_export.argtypes = [vp, i32, vp, i64]
+    lib.duo_device_status.argtypes = [vp]
+    lib.duo_strerror.argtypes = [i32]
+    lib.duo_strerror.restype = ctypes.c_char_p
+    for name in ("duo_pack", "duo_sparsify", "duo_spmspv", "duo_spmspv_multi", "duo_free",
+                 "duo_packed_query", "duo_packed_export", "duo_device_status", "duo_abi_version"):
+        getattr(lib, name).restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def duo_strerror(code: int) -> str:
+    return load_library().duo_strerror(int(code)).decode()
+
+
+def _stream_ptr(stream) -> int | None:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _ptr(t: torch.Tensor | None):
+    return None if t is None else t.data_ptr()
+
+
+def _check(rc: int, what: str):
+    if rc != DUO_OK:
+        raise DuoError(rc, what)
+
+
+@dataclass
+class PackedInfo:
+    fmt: int
+    version: int
+    magic: int
+    seg_rows: int
+    out: int
+    inp: int
+    nseg: int
+    nnz: int
+    index_dev: int
+    index_bytes: int
+    aux_dev: int
+    aux_bytes: int
+    data_dev: int
+    data_bytes: int
+
+
+class Packed:
+    """Owner of a duo_packed handle (freed by :meth:`free` or on collection)."""
+
+    def __init__(self, handle: int, out: int, inp: int, fmt: int):
+        self._h = handle
+        self.out, self.inp, self.fmt = out, inp, fmt
+
+    @property
+    def handle(self) -> int:
+        if not self._h:
+            raise DuoError(DUO_EINVAL, "handle already freed")
+        return self._h
+
+    def query(self) -> PackedInfo:
+        info = _Info()
+        _check(load_library().duo_packed_query(self.handle, ctypes.byref(info)), "duo_packed_query")
+        return PackedInfo(*[getattr(info, f[0]) or 0 for f in _Info._fields_])
+
+    def free(self):
+        if self._h:
+            h, self._h = self._h, None
+            _check(load_library().duo_free(h), "duo_free")
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def duo_pack(W: torch.Tensor, fmt="bitmask", stream=None) -> Packed:
+    """Packs an O x I fp16 CUDA weight (pruned entries zero); see duo_pack in
+    include/duo.h.  Row-major with unit column stride; any row stride."""
+    if W.dtype != torch.float16 or W.dim() != 2 or not W.is_cuda:
+        raise DuoError(DUO_EINVAL, "duo_pack needs a 2-D fp16 CUDA tensor")
+    if W.stride(1) != 1:
+        raise DuoError(DUO_EINVAL, "duo_pack needs unit column stride")
+    f = FORMATS[fmt] if isinstance(fmt, str) else int(fmt)
+    h = ctypes.c_void_p()
+    O, I = W.shape
+    _check(load_library().duo_pack(W.data_ptr(), O, I, W.stride(0), f, _stream_ptr(stream),
+                                   ctypes.byref(h)), "duo_pack")
+    return Packed(h.value, O, I, f)
+
+
+def duo_sparsify(x: torch.Tensor, k: int, kept_idx: torch.Tensor | None = None,
+                 kept_val: torch.Tensor | None = None, stream=None):
+    """Kept channel ids (uint16 bits in an int16 tensor, ascending) and their
+    fp16 values for the k largest |x| (§3)."""
+    I = x.numel()
+    if kept_idx is None:
+        kept_idx = torch.empty(k, dtype=torch.int16, device=x.device)
+    if kept_val is None:
+        kept_val = torch.empty(k, dtype=torch.float16, device=x.device)
+    _check(load_library().duo_sparsify(_ptr(x), I, int(k), _ptr(kept_idx), _ptr(kept_val),
+                                       _stream_ptr(stream)), "duo_sparsify")
+    return kept_idx, kept_val
+
+
+def duo_spmspv(h: Packed, x: torch.Tensor | None, k: int, kept_idx=None, kept_val=None,
+               y: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """y = W (x ⊙ m^x) (§3): fused selection when kept_idx/kept_val are None."""
+    if y is None:
+        dev = (x if x is not None else kept_idx).device
+        y = torch.empty(h.out, dtype=torch.float32, device=dev)
+    _check(load_library().duo_spmspv(h.handle, _ptr(x), _ptr(kept_idx), _ptr(kept_val), int(k),
+                                     _ptr(y), _stream_ptr(stream)), "duo_spmspv")
+    return y
+
+
+def duo_spmspv_multi(hs, x: torch.Tensor | None, k: int, kept_idx=None, kept_val=None,
+                     ys=None, stream=None):
+    """n products sharing one sparse input (q/k/v, gate/up) in one launch."""
+    n = len(hs)
+    if ys is None:
+        dev = (x if x is not None else kept_idx).device
+        ys = [torch.empty(h.out, dtype=torch.float32, device=dev) for h in hs]
+    harr = (ctypes.c_void_p * n)(*[h.handle for h in hs])
+    yarr = (ctypes.c_void_p * n)(*[y.data_ptr() for y in ys])
+    _check(load_library().duo_spmspv_multi(harr, n, _ptr(x), _ptr(kept_idx), _ptr(kept_val),
+                                           int(k), yarr, _stream_ptr(stream)), "duo_spmspv_multi")
+    return ys
+
+
+def duo_free(h: Packed):
+    h.free()
+
+
+def duo_device_status(stream=None) -> int:
+    return load_library().duo_device_status(_stream_ptr(stream))
+
+
+def packed_bytes(h: Packed):
+    """Copies a handle's index / aux / data buffers to host numpy uint8
+    arrays through duo_packed_export (byte-level parity checks, saving)."""
+    import numpy as np
+    info = h.query()
+    lib = load_library()
+    out = []
+    for which, n in ((0, info.index_bytes), (1, info.aux_bytes), (2, info.data_bytes)):
+        buf = np.zeros(n, dtype=np.uint8)
+        _check(lib.duo_packed_export(h.handle, which, buf.ctypes.data if n else None, n),
+               "duo_packed_export")
+        out.append(buf)
+    return (info, *out)

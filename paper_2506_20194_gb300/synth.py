@@ -55,7 +55,19 @@ def gen_weight(O: int, I: int, sigma: float, pw: float, prune: str, seed_w: int,
     elif prune == "magnitude":
         keep = torch.ones((O, I), dtype=torch.bool, device=device)
         a = w.abs().to(torch.float32)
-        for b0 in range(0, I, PRUNE_BLOCK):
+        nfull = I // PRUNE_BLOCK
+        if nfull:
+            # all full blocks at once: [nb, O*128], flat index r*128 + c
+            blk = a[:, : nfull * PRUNE_BLOCK].reshape(O, nfull, PRUNE_BLOCK).permute(1, 0, 2)
+            blk = blk.reshape(nfull, O * PRUNE_BLOCK)
+            n_prune = int(round(pw * O * PRUNE_BLOCK))
+            if n_prune:
+                order = torch.sort(blk, dim=1, stable=True).indices[:, :n_prune]
+                kb = torch.ones_like(blk, dtype=torch.bool)
+                kb.scatter_(1, order, False)
+                keep[:, : nfull * PRUNE_BLOCK] = kb.view(nfull, O, PRUNE_BLOCK).permute(1, 0, 2) \
+                    .reshape(O, nfull * PRUNE_BLOCK)
+        for b0 in range(nfull * PRUNE_BLOCK, I, PRUNE_BLOCK):
             b1 = min(I, b0 + PRUNE_BLOCK)
             blk = a[:, b0:b1].reshape(-1)
             n_prune = int(round(pw * blk.numel()))

@@ -1,0 +1,109 @@
+"""C ABI checks that need no GPU: the library builds and loads, exports every
+function include/duo.h declares, and rejects invalid arguments on the host
+before any device work (no pointer below is ever dereferenced)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "duo.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2506_20194_gb300.build import build_library
+    build_library()
+    from paper_2506_20194_gb300 import duo
+    return duo.load_library()
+
+
+def _declared_functions():
+    txt = open(HEADER).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(duo_\w+)\s*\(", txt, flags=re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared_functions()
+    for n in ("duo_pack", "duo_sparsify", "duo_spmspv", "duo_spmspv_multi", "duo_free",
+              "duo_strerror", "duo_packed_query", "duo_packed_export", "duo_device_status",
+              "duo_abi_version"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for n in _declared_functions():
+        assert hasattr(lib, n), f"{n} declared in duo.h but not exported"
+
+
+def test_abi_version_and_strerror(lib):
+    assert lib.duo_abi_version() == 1
+    from paper_2506_20194_gb300 import duo
+    for code in (0, -1, -2, -3, -4, -5, -6):
+        assert duo.duo_strerror(code) and duo.duo_strerror(code) != "unknown status code"
+    assert duo.duo_strerror(-99) == "unknown status code"
+
+
+FAKE = 0x10000   # never dereferenced: validation rejects every call first
+
+
+def test_pack_argument_validation(lib):
+    h = ctypes.c_void_p()
+    EINVAL, ERANGE = -1, -4
+    assert lib.duo_pack(None, 4, 4, 4, 1, None, ctypes.byref(h)) == EINVAL
+    assert lib.duo_pack(FAKE, 4, 4, 4, 1, None, None) == EINVAL
+    assert lib.duo_pack(FAKE, 0, 4, 4, 1, None, ctypes.byref(h)) == EINVAL
+    assert lib.duo_pack(FAKE, 4, 0, 4, 1, None, ctypes.byref(h)) == EINVAL
+    assert lib.duo_pack(FAKE, 4, 8, 4, 1, None, ctypes.byref(h)) == EINVAL     # ldw < in
+    assert lib.duo_pack(FAKE, 4, 4, 4, 7, None, ctypes.byref(h)) == EINVAL     # fmt
+    assert lib.duo_pack(FAKE + 1, 4, 4, 4, 1, None, ctypes.byref(h)) == EINVAL  # alignment
+    assert lib.duo_pack(FAKE, 4, 65536, 65536, 1, None, ctypes.byref(h)) == ERANGE
+    assert lib.duo_pack(FAKE, 70000, 4, 4, 0, None, ctypes.byref(h)) == ERANGE  # IDX16 rows
+    assert h.value is None
+    # Passes host validation; without a GPU (or with a non-device pointer)
+    # the call still fails cleanly.
+    assert lib.duo_pack(FAKE, 4, 4, 4, 1, None, ctypes.byref(h)) in (-1, -3)
+    assert h.value is None
+
+
+def test_sparsify_argument_validation(lib):
+    EINVAL = -1
+    assert lib.duo_sparsify(None, 8, 2, FAKE, FAKE, None) == EINVAL
+    assert lib.duo_sparsify(FAKE, 0, 0, FAKE, FAKE, None) == EINVAL
+    assert lib.duo_sparsify(FAKE, 65536, 2, FAKE, FAKE, None) == EINVAL
+    assert lib.duo_sparsify(FAKE, 8, 9, FAKE, FAKE, None) == EINVAL
+    assert lib.duo_sparsify(FAKE, 8, -1, FAKE, FAKE, None) == EINVAL
+    assert lib.duo_sparsify(FAKE, 8, 2, None, FAKE, None) == EINVAL
+    assert lib.duo_sparsify(FAKE + 1, 8, 2, FAKE, FAKE, None) == EINVAL
+
+
+def test_spmspv_rejects_dead_or_fake_handles(lib):
+    EINVAL = -1
+    assert lib.duo_spmspv(None, FAKE, None, None, 2, FAKE, None) == EINVAL
+    assert lib.duo_spmspv(FAKE, FAKE, None, None, 2, FAKE, None) == EINVAL   # not a live handle
+    assert lib.duo_spmspv(FAKE, FAKE, FAKE, None, 2, FAKE, None) == EINVAL   # half a kept list
+    arr = (ctypes.c_void_p * 5)(FAKE, FAKE, FAKE, FAKE, FAKE)
+    assert lib.duo_spmspv_multi(arr, 5, FAKE, None, None, 2, arr, None) == EINVAL   # n > 4
+    assert lib.duo_spmspv_multi(arr, 0, FAKE, None, None, 2, arr, None) == EINVAL
+
+
+def test_free_and_query_reject_non_handles(lib):
+    assert lib.duo_free(None) == 0
+    assert lib.duo_free(FAKE) == -1
+    from paper_2506_20194_gb300 import duo
+    info = duo._Info()
+    assert lib.duo_packed_query(FAKE, ctypes.byref(info)) == -1
+    assert lib.duo_packed_export(FAKE, 0, FAKE, 16) == -1
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    import paper_2506_20194_gb300.duo as duo
+    saved = duo._lib
+    try:
+        duo._lib = None
+        with pytest.raises(RuntimeError):
+            duo.load_library(str(tmp_path / "missing.so"))
+    finally:
+        duo._lib = saved
