@@ -154,48 +154,50 @@ def required_bytes_layer(duo, shape, layer, px):
 
 def stage_calls(duo, shape, layer, px):
     def run():
-        for st, src in zip(STAGES, STAGE_SRC):
-            k = k_of(shape.I(st[0]), px)
-            if len(st) == 1:
-                duo.duo_spmspv(layer["h"][st[0]], layer["x"][src], k, y=layer["y"][st[0]])
-            else:
-                duo.duo_spmspv_multi([layer["h"][p] for p in st], layer["x"][src], k,
-                                     ys=[layer["y"][p] for p in st])
+        for si in range(len(STAGES)):
+            stage_call(duo, shape, layer, px, si)
     return run
 
 
-def capture_rotation(duo, shape, layers, px, with_events):
-    """One CUDA graph replaying every layer once (L steps), with timing
-    events around each stage launch when supported."""
-    events = None
-    if with_events:
-        try:
-            events = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(len(STAGES) + 1)]
-                      for _ in layers]
-        except TypeError:
-            events = None
+def capture(fn):
+    """Captures fn() into a CUDA graph after one eager warm-up run."""
     s = torch.cuda.Stream()
     s.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(s):           # warm the launch path (attributes, module load)
-        for layer in layers:
-            stage_calls(duo, shape, layer, px)()
+        fn()
     torch.cuda.current_stream().wait_stream(s)
     torch.cuda.synchronize()
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g):
-        for li, layer in enumerate(layers):
-            for si, (st, src) in enumerate(zip(STAGES, STAGE_SRC)):
-                if events is not None:
-                    events[li][si].record()
-                k = k_of(shape.I(st[0]), px)
-                if len(st) == 1:
-                    duo.duo_spmspv(layer["h"][st[0]], layer["x"][src], k, y=layer["y"][st[0]])
-                else:
-                    duo.duo_spmspv_multi([layer["h"][p] for p in st], layer["x"][src], k,
-                                         ys=[layer["y"][p] for p in st])
-            if events is not None:
-                events[li][len(STAGES)].record()
-    return g, events
+        fn()
+    return g
+
+
+def stage_call(duo, shape, layer, px, si):
+    st, src = STAGES[si], STAGE_SRC[si]
+    k = k_of(shape.I(st[0]), px)
+    if len(st) == 1:
+        duo.duo_spmspv(layer["h"][st[0]], layer["x"][src], k, y=layer["y"][st[0]])
+    else:
+        duo.duo_spmspv_multi([layer["h"][p] for p in st], layer["x"][src], k,
+                             ys=[layer["y"][p] for p in st])
+
+
+def capture_rotation(duo, shape, layers, px):
+    """One CUDA graph replaying every layer once (L steps, 4 launches each)."""
+    def fn():
+        for layer in layers:
+            for si in range(len(STAGES)):
+                stage_call(duo, shape, layer, px, si)
+    return capture(fn)
+
+
+def capture_stage(duo, shape, layers, px, si):
+    """One CUDA graph launching stage si of every layer (L launches)."""
+    def fn():
+        for layer in layers:
+            stage_call(duo, shape, layer, px, si)
+    return capture(fn)
 
 
 def time_graph(g, reps):
@@ -344,7 +346,7 @@ def run_ours(args):
     breq_mean = float(np.mean([b for b, _ in breq_layers]))
     stage_b = np.mean(np.array([ps for _, ps in breq_layers]), axis=0)
 
-    g, events = capture_rotation(duo, shape, layers, args.px, with_events=True)
+    g = capture_rotation(duo, shape, layers, args.px)
     reps_w = max(1, math.ceil(args.warmup / L))
     reps = max(1, args.steps // L)
     steps_timed = reps * L
@@ -360,25 +362,24 @@ def run_ours(args):
     us_layer = t / steps_timed * 1e6
     value = breq_mean * steps_timed * world / t / 1e9
 
-    # per-stage kernel durations from the in-graph events of the last replay
-    stage_us = None
-    if events is not None:
-        try:
-            st_ms = np.array([[events[l][s].elapsed_time(events[l][s + 1]) for s in range(len(STAGES))]
-                              for l in range(L)])
-            stage_us = st_ms.mean(axis=0) * 1e3
-        except Exception:
-            stage_us = None
+    # Average launch duration of the fused kernel per stage: a graph of that
+    # stage's launch for every layer, timed with CUDA events on the stream.
+    stage_us = []
+    for si in range(len(STAGES)):
+        gs = capture_stage(duo, shape, layers, args.px, si)
+        time_graph(gs, 3)
+        r = max(3, min(reps, 500))
+        stage_us.append(time_graph(gs, r) / (r * L) * 1e6)
+        del gs
+    stage_us = np.array(stage_us)
     peak, peak_kind = peaks()
-    if stage_us is not None:
-        achieved = float(stage_b.sum() / (stage_us.sum() * 1e-6) / 1e9)
-    else:
-        achieved = breq_mean / (us_layer * 1e-6) / 1e9
+    achieved = float(stage_b.sum() / (stage_us.sum() * 1e-6) / 1e9)
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "peak_kind": peak_kind, "traffic": None,
                 "kernel": "cmb_spmspv_kernel<fused>",
                 "per_launch_bytes": [float(b) for b in stage_b],
-                "per_launch_us": None if stage_us is None else [float(u) for u in stage_us]}
+                "per_launch_us": [float(u) for u in stage_us],
+                "per_launch_GBps": [float(b / (u * 1e-6) / 1e9) for b, u in zip(stage_b, stage_us)]}
 
     # end to end through the public API with host buffers
     e2e = run_e2e(duo, shape, layers, args, breq_mean)
@@ -389,7 +390,7 @@ def run_ours(args):
     sweep = {}
     if not args.no_sweep:
         for px in (0, 25, 50, 70):
-            gs, _ = capture_rotation(duo, shape, layers, px, with_events=False)
+            gs = capture_rotation(duo, shape, layers, px)
             time_graph(gs, 5)
             r = max(1, min(reps, 400))
             ts = time_graph(gs, r)

@@ -117,9 +117,9 @@ int duo_sparsify(const void* x_fp16_dev, int64_t in, int64_t k,
  *   listed  : kept_idx_dev (uint16[k], distinct ids < in, any order) and
  *             kept_val_fp16_dev (fp16[k]) give the sparse input directly;
  *             x_fp16_dev is ignored and may be NULL.
- *   y_dev   : device fp32[O], 16-byte aligned; fully overwritten (the call
- *             zeroes it on `stream` first).  Summation order is not fixed,
- *             so y is reproducible only to fp32 rounding.
+ *   k == 0  : y = 0; the input pointers are not read and may be NULL.
+ *   y_dev   : device fp32[O], 16-byte aligned; fully overwritten.  Summation
+ *             order is not fixed, so y is reproducible only to fp32 rounding.
  * Errors: DUO_EINVAL (NULL, alignment, k, dead handle), DUO_ECUDA.
  */
 /* Concurrency: calls whose first handle is the same must be ordered on the
@@ -166,7 +166,8 @@ int duo_packed_query(const duo_packed* h, duo_packed_info* info);
 /* Copies one buffer of a live handle to host memory (synchronous), e.g. to
  * save a packed weight or to compare its bytes with a reference packer.
  *   which : 0 = index, 1 = aux, 2 = data (as described by duo_packed_info).
- *   dst_host, bytes : host destination; bytes must equal the buffer size.
+ *   dst_host, bytes : host destination; bytes must equal the buffer size
+ *                     (dst_host may be NULL when that size is 0).
  * Errors: DUO_EINVAL (dead handle, which, NULL dst, size mismatch), DUO_ECUDA. */
 int duo_packed_export(const duo_packed* h, int which, void* dst_host, int64_t bytes);
 

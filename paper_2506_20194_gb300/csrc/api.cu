@@ -8,7 +8,7 @@
 
 #include <cuda_runtime.h>
 
-#include "../../include/duo.h"
+#include "duo.h"
 #include "duo_launch.h"
 
 namespace {
@@ -31,6 +31,7 @@ struct duo_packed {
   void* data;
   int64_t data_bytes;
   unsigned int* sync;  // BITMASK: 2-word grid barrier of the spMspV kernel
+  int max_record;      // BITMASK: bytes of the largest record
 };
 
 namespace {
@@ -154,7 +155,7 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
   cudaError_t e = duo_malloc(reinterpret_cast<void**>(&cnt_js), sizeof(uint32_t) * in * S);
   if (e != cudaSuccess) return map_err(e);
   scratch.add(cnt_js);
-  e = duo_malloc(reinterpret_cast<void**>(&totals), 2 * sizeof(unsigned long long));
+  e = duo_malloc(reinterpret_cast<void**>(&totals), 3 * sizeof(unsigned long long));
   if (e != cudaSuccess) return map_err(e);
   scratch.add(totals);
 
@@ -178,7 +179,7 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
     return code;
   };
 
-  unsigned long long host_tot[2] = {0, 0};
+  unsigned long long host_tot[3] = {0, 0, 0};
   if (fmt == DUO_FMT_BITMASK) {
     h->nseg = S;
     h->index_bytes = (int64_t)sizeof(uint32_t) * (in * S + 1);
@@ -197,6 +198,7 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
     if (e != cudaSuccess) return fail(map_err(e));
     if (host_tot[0] >= (1ull << 32)) return fail(DUO_ERANGE);
     h->data_bytes = (int64_t)host_tot[0] * 16;
+    h->max_record = (int)((128 + 2 * host_tot[2] + 15) / 16 * 16);
     e = duo_malloc(&data, (size_t)h->data_bytes);
     if (e != cudaSuccess) return fail(map_err(e));
     e = cudaMemsetAsync(data, 0, (size_t)h->data_bytes, st);
@@ -215,7 +217,7 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
     e = duo::launch_idx16_offsets(cnt_js, in, (int)S, static_cast<uint32_t*>(aux),
                                   static_cast<uint64_t*>(index), totals, st);
     if (e != cudaSuccess) return fail(map_err(e));
-    e = cudaMemcpyAsync(host_tot, totals, sizeof(host_tot), cudaMemcpyDeviceToHost, st);
+    e = cudaMemcpyAsync(host_tot, totals, 2 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return fail(map_err(e));
     h->data_bytes = (int64_t)host_tot[0];
@@ -263,8 +265,10 @@ static int spmspv_common(const duo_packed* const* hs, int n, const void* x, cons
                          const void* kval, int64_t k, float* const* ys, void* stream) {
   if (hs == nullptr || ys == nullptr || n < 1 || n > duo::kMaxProblems) return DUO_EINVAL;
   const bool listed = kidx != nullptr || kval != nullptr;
-  if (listed && (kidx == nullptr || kval == nullptr)) return DUO_EINVAL;
-  if (!listed && x == nullptr) return DUO_EINVAL;
+  if (k != 0) {   // with k == 0 nothing is read: y = 0 whatever the input pointers
+    if (listed && (kidx == nullptr || kval == nullptr)) return DUO_EINVAL;
+    if (!listed && x == nullptr) return DUO_EINVAL;
+  }
   if (!aligned(x, 2) || !aligned(kidx, 2) || !aligned(kval, 2)) return DUO_EINVAL;
   for (int p = 0; p < n; ++p) {
     if (hs[p] == nullptr || ys[p] == nullptr) return DUO_EINVAL;
@@ -299,6 +303,8 @@ static int spmspv_common(const duo_packed* const* hs, int n, const void* x, cons
     a.kidx = listed ? kidx : nullptr;
     a.kval = listed ? static_cast<const uint16_t*>(kval) : nullptr;
     a.bar = hs[0]->sync;
+    a.slot_bytes = 0;
+    for (int p = 0; p < n; ++p) a.slot_bytes = hs[p]->max_record > a.slot_bytes ? hs[p]->max_record : a.slot_bytes;
     for (int p = 0; p < n; ++p) {
       a.p[p].data = static_cast<const uint8_t*>(hs[p]->data);
       a.p[p].off = static_cast<const uint32_t*>(hs[p]->index);
@@ -379,7 +385,8 @@ int duo_packed_query(const duo_packed* h, duo_packed_info* info) {
 }
 
 int duo_packed_export(const duo_packed* h, int which, void* dst_host, int64_t bytes) {
-  if (h == nullptr || dst_host == nullptr || !is_live(h)) return DUO_EINVAL;
+  if (h == nullptr || !is_live(h)) return DUO_EINVAL;
+  if (dst_host == nullptr && bytes != 0) return DUO_EINVAL;
   const void* src = nullptr;
   int64_t n = 0;
   switch (which) {

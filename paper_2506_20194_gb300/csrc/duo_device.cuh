@@ -103,6 +103,11 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
+// L2 prefetch of [src, src + bytes) (16-byte aligned, bytes % 16 == 0).
+__device__ __forceinline__ void prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 __device__ __forceinline__ uint64_t policy_evict_first() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
@@ -113,6 +118,22 @@ __device__ __forceinline__ unsigned int ld_acquire_gpu(const unsigned int* p) {
   unsigned int v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
+}
+
+__device__ __forceinline__ unsigned int ld_relaxed_gpu(const unsigned int* p) {
+  unsigned int v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ unsigned int atom_add_acq_rel_gpu(unsigned int* p, unsigned int v) {
+  unsigned int old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
+__device__ __forceinline__ void red_add_release_gpu(unsigned int* p, unsigned int v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
@@ -197,131 +218,259 @@ __device__ inline void load_x_to_smem(uint16_t* xs, const uint16_t* x, int I) {
   }
 }
 
+constexpr int SEL_BINS = 4096;   // histogram of key >> 3
+
+// Shared state of the selection.
 struct SelShared {
-  uint32_t hist[256];
-  uint32_t wsum[32];
-  int b1;
-  uint32_t above1;
-  uint32_t T;
-  int q;
+  uint32_t hist[SEL_BINS];
+  uint32_t wtot[32];     // per-warp partial sums
+  uint32_t sub[32][4];   // per-warp counts of key & 7 inside the threshold bin (16-bit pairs)
+  uint32_t B;            // threshold bin
+  uint32_t aboveB;       // channels in bins above it
 };
+
+// Clears the histogram (before the __syncthreads that precedes select_topk).
+__device__ __forceinline__ void select_clear(SelShared* sh) {
+  uint4* h = reinterpret_cast<uint4*>(sh->hist);
+  for (int i = threadIdx.x; i < SEL_BINS / 4; i += blockDim.x) h[i] = make_uint4(0u, 0u, 0u, 0u);
+}
 
 // Exact top-k by magnitude (§3): keeps the k channels with the largest
 // |x_j|, ties to the lower index.  The key of x_j is its fp16 bit pattern
 // with the sign cleared; for IEEE fp16 this integer order equals the order of
-// |x_j| (NaN patterns sort above Inf).  Two radix passes (8 high key bits,
-// then 7 low bits) find the threshold key T and the number q of channels
-// with key == T to keep (the q lowest-indexed ones).
+// |x_j| (NaN patterns sort above Inf).
 //
-// Output, in shared memory, for nw = ceil(I/32) words:
-//   kb[w]  kept-channel bitmap (bit b <-> channel 32w+b),
-//   kp[w]  number of kept channels before word w, kp[nw] = k.
-// eqw is nw words of scratch.  All threads of the block must call it.
-__device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t* kb, uint32_t* kp,
-                                   uint32_t* eqw, SelShared* sh) {
+//  1. histogram of key >> 3 (4096 bins, shared-memory atomics; a thread's
+//     keys are in registers);
+//  2. suffix scan of the histogram (512 threads x 8 bins) to find the bin B
+//     where the count from the top reaches k;
+//  3. per-warp counts of the 8 keys inside bin B (warp reductions, no
+//     atomics) give the threshold key T and the count above it; the
+//     q = k - count(key > T) lowest-indexed channels with key == T are kept;
+//  4. every thread builds the "above T" / "equal to T" masks of its own
+//     32-channel words from 16-byte loads of x, a block exclusive scan of the
+//     packed counts orders the words, and the thread writes kb[w] (kept
+//     bitmap, bit b <-> channel 32w+b) and kp[w] (kept channels before word
+//     w; kp[nw] = k);
+//  5. warps emit klist[r] (channel of kept rank r, ascending) and kvals[r]
+//     (its fp16 bits) word by word, lane = bit, if requested.
+// Shared-memory accesses are arranged to be bank-conflict free (rotated
+// 16-byte chunks).
+//
+// select_keys_load() runs first (it also writes xs, the fp16 bits of x, to
+// shared memory; xs needs room for a multiple of 32 entries), then
+// select_clear(), then a __syncthreads.  All threads of the block take part
+// (blockDim.x >= 512, a multiple of 32); it ends with a __syncthreads.
+constexpr int SEL_MAXKEYS = 32;   // keys per thread kept in registers
+constexpr uint32_t KEY_NONE = 0xFFFFu;
+
+struct SelKeys {
+  uint32_t key[SEL_MAXKEYS];
+  int n;   // keys held (channels tid, tid + blockDim, ...)
+};
+
+__device__ __forceinline__ void select_keys_load(SelKeys& K, const uint16_t* __restrict__ x,
+                                                 uint16_t* xs, int I) {
+  const int nt = blockDim.x;
+  K.n = (I - (int)threadIdx.x + nt - 1) / nt;
+  if (K.n <= SEL_MAXKEYS) {
+#pragma unroll
+    for (int r = 0; r < SEL_MAXKEYS; ++r) {
+      const int j = threadIdx.x + r * nt;
+      uint32_t v = KEY_NONE;
+      if (j < I) {
+        const uint16_t b = x[j];
+        xs[j] = b;
+        v = b & 0x7FFFu;
+      }
+      K.key[r] = v;
+    }
+  } else {
+    load_x_to_smem(xs, x, I);
+  }
+}
+
+template <typename F>
+__device__ __forceinline__ void for_each_key(const SelKeys& K, const uint16_t* xs, int I, F f) {
+  if (K.n <= SEL_MAXKEYS) {
+#pragma unroll
+    for (int r = 0; r < SEL_MAXKEYS; ++r)
+      if (K.key[r] != KEY_NONE) f(K.key[r]);
+  } else {
+    for (int j = threadIdx.x; j < I; j += blockDim.x) f((uint32_t)(xs[j] & 0x7FFFu));
+  }
+}
+
+// Masks of the channels of word w (32 channels) above T and equal to T.  The
+// four 16-byte chunks are read in an order rotated by (w >> 1) so that the
+// eight threads of a quarter warp (consecutive words) hit distinct banks.
+__device__ __forceinline__ void word_masks(const uint16_t* xs, int I, int w, bool all, bool none,
+                                           uint32_t T, uint32_t& gt, uint32_t& eq) {
+  const uint4* p = reinterpret_cast<const uint4*>(xs + 32 * w);
+  const int rot = (w >> 1) & 3;
+  gt = 0u;
+  eq = 0u;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int ci = (i + rot) & 3;
+    const uint4 c = p[ci];
+    const uint32_t v[4] = {c.x, c.y, c.z, c.w};
+#pragma unroll
+    for (int h = 0; h < 8; ++h) {
+      const uint32_t key = (v[h >> 1] >> (16 * (h & 1))) & 0x7FFFu;
+      const int b = 8 * ci + h;
+      gt |= (uint32_t)(key > T) << b;
+      eq |= (uint32_t)(key == T) << b;
+    }
+  }
+  const int valid = min(32, I - 32 * w);
+  const uint32_t vmask = valid >= 32 ? FULL_MASK : ((1u << valid) - 1u);
+  if (all) { gt = FULL_MASK; eq = 0u; }
+  if (none) { gt = 0u; eq = 0u; }
+  gt &= vmask;
+  eq &= vmask;
+}
+
+__device__ inline void select_topk(const SelKeys& K, const uint16_t* xs, int I, int k, uint32_t* kb,
+                                   uint32_t* kp, uint16_t* klist, uint16_t* kvals, SelShared* sh) {
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, wid = tid >> 5;
   const int nwarps = nt >> 5;
   const int nw = (I + 31) >> 5;
-  if (k <= 0 || k >= I) {
-    for (int w = tid; w < nw; w += nt) {
-      const int rem = I - 32 * w;
-      const uint32_t full = rem >= 32 ? FULL_MASK : ((1u << rem) - 1u);
-      kb[w] = k > 0 ? full : 0u;
-    }
+  const bool all = k >= I, none = k <= 0;
+  uint32_t T = 0u;
+  int q = 0;
+  if (!all && !none) {
+    // 1. histogram of the high 12 key bits
+    for_each_key(K, xs, I, [&](uint32_t key) { atomicAdd(&sh->hist[key >> 3], 1u); });
     __syncthreads();
-  } else {
-    for (int i = tid; i < 256; i += nt) sh->hist[i] = 0u;
-    __syncthreads();
-    for (int j = tid; j < I; j += nt) atomicAdd(&sh->hist[(xs[j] & 0x7FFFu) >> 7], 1u);
-    __syncthreads();
-    if (wid == 0) {
-      uint32_t c[8], s = 0;
+    // 2. suffix scan: thread t < 512 owns bins [8t, 8t + 8)
+    uint32_t c[8], s = 0, incl = 0;
+    if (tid < 512) {
+      const uint4* hp = reinterpret_cast<const uint4*>(sh->hist) + 2 * tid;
+      const int r = (tid >> 2) & 1;   // rotated halves: conflict-free quarter warps
+      const uint4 ha = hp[r], hb = hp[r ^ 1];
+      const uint4 h0 = r ? hb : ha, h1 = r ? ha : hb;
+      c[0] = h0.x; c[1] = h0.y; c[2] = h0.z; c[3] = h0.w;
+      c[4] = h1.x; c[5] = h1.y; c[6] = h1.z; c[7] = h1.w;
 #pragma unroll
-      for (int q = 0; q < 8; ++q) { c[q] = sh->hist[8 * lane + q]; s += c[q]; }
-      uint32_t sfx = s;   // inclusive suffix sum over lanes >= lane
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t t = __shfl_down_sync(FULL_MASK, sfx, o);
-        if (lane + o < 32) sfx += t;
-      }
-      const uint32_t above = sfx - s;
-      if (above < (uint32_t)k && (uint32_t)k <= sfx) {
-        uint32_t acc = above;
-        int b = 8 * lane;
-        for (int q = 7; q >= 0; --q) {
-          if (acc + c[q] >= (uint32_t)k) { b = 8 * lane + q; break; }
-          acc += c[q];
-        }
-        sh->b1 = b;
-        sh->above1 = acc;
-      }
-    }
-    __syncthreads();
-    const uint32_t b1 = (uint32_t)sh->b1;
-    const uint32_t above1 = sh->above1;
-    for (int i = tid; i < 128; i += nt) sh->hist[i] = 0u;
-    __syncthreads();
-    for (int j = tid; j < I; j += nt) {
-      const uint32_t key = xs[j] & 0x7FFFu;
-      if ((key >> 7) == b1) atomicAdd(&sh->hist[key & 127u], 1u);
-    }
-    __syncthreads();
-    if (wid == 0) {
-      const uint32_t need = (uint32_t)k - above1;
-      uint32_t c[4], s = 0;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) { c[q] = sh->hist[4 * lane + q]; s += c[q]; }
-      uint32_t sfx = s;
+      for (int i = 0; i < 8; ++i) s += c[i];
+      incl = s;   // suffix over lanes >= lane inside the warp
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t t = __shfl_down_sync(FULL_MASK, sfx, o);
-        if (lane + o < 32) sfx += t;
+        const uint32_t t = __shfl_down_sync(FULL_MASK, incl, o);
+        if (lane + o < 32) incl += t;
       }
-      const uint32_t above = sfx - s;
-      if (above < need && need <= sfx) {
-        uint32_t acc = above;
-        int b2 = 4 * lane;
-        for (int q = 3; q >= 0; --q) {
-          if (acc + c[q] >= need) { b2 = 4 * lane + q; break; }
-          acc += c[q];
+      if (lane == 0) sh->wtot[wid] = incl;
+    }
+    __syncthreads();
+    if (tid < 512) {
+      uint32_t above_w = (lane > wid && lane < 16) ? sh->wtot[lane] : 0u;
+      above_w = __reduce_add_sync(FULL_MASK, above_w);
+      const uint32_t hi = above_w + incl;   // channels in bins >= 8*tid
+      const uint32_t lo = hi - s;           // channels in bins >= 8*tid + 8
+      if (lo < (uint32_t)k && (uint32_t)k <= hi) {
+        uint32_t acc = lo;
+        int b = 0;
+#pragma unroll
+        for (int i = 7; i >= 0; --i) {
+          if (acc + c[i] >= (uint32_t)k) { b = i; break; }
+          acc += c[i];
         }
-        sh->T = b1 * 128u + (uint32_t)b2;
-        sh->q = (int)(need - acc);
+        sh->B = 8u * tid + (uint32_t)b;
+        sh->aboveB = acc;
       }
     }
     __syncthreads();
-    const uint32_t T = sh->T;
-    const int q = sh->q;
+    // 3. the 8 keys of bin B: per-thread counts in 16-bit fields, reduced
+    //    per warp, then summed over warps
+    const uint32_t B = sh->B;
+    uint32_t cnt[4] = {0u, 0u, 0u, 0u};
+    for_each_key(K, xs, I, [&](uint32_t key) {
+      if ((key >> 3) == B) {
+        const uint32_t low = key & 7u;
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          cnt[v] += (low == 2u * v) ? 1u : 0u;
+          cnt[v] += (low == 2u * v + 1u) ? 0x10000u : 0u;
+        }
+      }
+    });
+#pragma unroll
+    for (int v = 0; v < 4; ++v) cnt[v] = __reduce_add_sync(FULL_MASK, cnt[v]);
+    if (lane == 0) {
+#pragma unroll
+      for (int v = 0; v < 4; ++v) sh->sub[wid][v] = cnt[v];
+    }
+    __syncthreads();
+    uint32_t tot4[4] = {0u, 0u, 0u, 0u};
+    for (int w2 = 0; w2 < nwarps; ++w2) {
+#pragma unroll
+      for (int v = 0; v < 4; ++v) tot4[v] += sh->sub[w2][v];
+    }
+    uint32_t above = sh->aboveB;
+    int b = -1;
+#pragma unroll
+    for (int v = 7; v >= 0; --v) {
+      const uint32_t cv = (tot4[v >> 1] >> (16 * (v & 1))) & 0xFFFFu;
+      if (b < 0) {
+        if (above + cv >= (uint32_t)k) b = v;
+        else above += cv;
+      }
+    }
+    if (b < 0) b = 0;
+    T = 8u * B + (uint32_t)b;
+    q = k - (int)above;
+  }
+  // 4. thread tid owns words [w0, w1)
+  const int per = (nw + nt - 1) / nt;
+  const int w0 = min(nw, tid * per), w1 = min(nw, w0 + per);
+  uint32_t packed = 0;   // greater-count | tie-count << 16 (each <= 65535)
+  for (int w = w0; w < w1; ++w) {
+    uint32_t gt, eq;
+    word_masks(xs, I, w, all, none, T, gt, eq);
+    kb[w] = gt;   // provisional: the masks are kept in kb / kp until ranked
+    kp[w] = eq;
+    packed += (uint32_t)__popc(gt) | ((uint32_t)__popc(eq) << 16);
+  }
+  const uint32_t inc = warp_inclusive_scan(packed, lane);
+  __syncthreads();   // wtot of step 2 is no longer read
+  if (lane == 31) sh->wtot[wid] = inc;
+  __syncthreads();
+  if (wid == 0) {
+    uint32_t t = lane < nwarps ? sh->wtot[lane] : 0u;
+    t = warp_inclusive_scan(t, lane);
+    sh->wtot[lane] = t;
+  }
+  __syncthreads();
+  const uint32_t base = (wid > 0 ? sh->wtot[wid - 1] : 0u) + inc - packed;
+  uint32_t gpre = base & 0xFFFFu, epre = base >> 16;
+  for (int w = w0; w < w1; ++w) {
+    const uint32_t gt = kb[w], eq = kp[w];
+    const int allowed = q - (int)epre;
+    uint32_t take = 0u;
+    if (allowed > 0 && eq != 0u)
+      take = allowed >= __popc(eq) ? eq : (eq & ((1u << select_bit(eq, allowed)) - 1u));
+    kb[w] = gt | take;
+    kp[w] = gpre + min(epre, (uint32_t)q);
+    gpre += __popc(gt);
+    epre += __popc(eq);
+  }
+  if (tid == 0) kp[nw] = all ? (uint32_t)I : (none ? 0u : (uint32_t)k);
+  __syncthreads();
+  // 5. warp-parallel emission of the kept list
+  if (klist != nullptr || kvals != nullptr) {
+    const uint32_t lt = (1u << lane) - 1u;
     for (int w = wid; w < nw; w += nwarps) {
-      const int j = 32 * w + lane;
-      const bool valid = j < I;
-      const uint32_t key = valid ? (xs[j] & 0x7FFFu) : 0u;
-      const uint32_t gt = __ballot_sync(FULL_MASK, valid && key > T);
-      const uint32_t eq = __ballot_sync(FULL_MASK, valid && key == T);
-      if (lane == 0) { kb[w] = gt; eqw[w] = eq; kp[w] = __popc(eq); }
-    }
-    __syncthreads();
-    block_exclusive_scan(kp, nw, sh->wsum);   // kp[w] = ties before word w
-    for (int w = tid; w < nw; w += nt) {
-      const int allowed = q - (int)kp[w];
-      const uint32_t eq = eqw[w];
-      if (allowed > 0 && eq != 0u) {
-        uint32_t take = eq;
-        if (allowed < __popc(eq)) {
-          uint32_t r = eq;
-          for (int t = 0; t < allowed; ++t) r &= r - 1u;
-          take = eq & ~r;
-        }
-        kb[w] |= take;
+      const uint32_t kbw = kb[w];
+      if ((kbw >> lane) & 1u) {
+        const uint32_t rank = kp[w] + __popc(kbw & lt);
+        const int j = 32 * w + lane;
+        if (klist != nullptr) klist[rank] = (uint16_t)j;
+        if (kvals != nullptr) kvals[rank] = xs[j];
       }
     }
     __syncthreads();
   }
-  for (int w = tid; w < nw; w += nt) kp[w] = __popc(kb[w]);
-  __syncthreads();
-  const uint32_t tot = block_exclusive_scan(kp, nw, sh->wsum);
-  if (tid == 0) kp[nw] = tot;
-  __syncthreads();
 }
 
 // Channel id of kept index i (0 <= i < kp[nw]) from the bitmap + prefix.

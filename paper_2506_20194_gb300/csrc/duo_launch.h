@@ -30,6 +30,8 @@ struct CmbArgs {
   const uint16_t* kval;  // listed mode: fp16 bits [k]
   unsigned int* bar;     // 2 words {count, generation} of a grid barrier, zero
                          // between launches; owned by the first handle
+  int slot_bytes;        // in: largest record of the launch's weights (bytes);
+                         // the launcher rounds it and picks the slot count
   int nslot;             // set by the launcher
 };
 
@@ -59,7 +61,8 @@ cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uin
 cudaError_t launch_pack_count(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
                               uint32_t* cnt_js, cudaStream_t st);
 // off[n] exclusive prefix (16-byte units) of the CMB record sizes;
-// totals[0] = total units (64-bit), totals[1] = total non-zeros.
+// totals[0] = total units (64-bit), totals[1] = total non-zeros,
+// totals[2] = largest per-record non-zero count.
 cudaError_t launch_cmb_offsets(const uint32_t* cnt_js, int64_t n, uint32_t* off,
                                unsigned long long* totals, cudaStream_t st);
 cudaError_t launch_cmb_scatter(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,

@@ -238,8 +238,19 @@ __global__ void __launch_bounds__(SCAN_THREADS) cmb_offsets_kernel(const uint32_
   chunked_scan(
       n, [&](int64_t i) { return (unsigned long long)cnt_js[i]; },
       [&](int64_t, unsigned long long) {}, &totals[1]);
+  // largest record non-zero count
+  __shared__ uint32_t wmax[SCAN_THREADS / 32];
+  uint32_t m = 0;
+  for (int64_t i = threadIdx.x; i < n; i += SCAN_THREADS) m = max(m, cnt_js[i]);
+  m = __reduce_max_sync(FULL_MASK, m);
+  if ((threadIdx.x & 31) == 0) wmax[threadIdx.x >> 5] = m;
   __syncthreads();
-  if (threadIdx.x == 0) off[n] = (uint32_t)totals[0];
+  if (threadIdx.x == 0) {
+    uint32_t mm = 0;
+    for (int w = 0; w < SCAN_THREADS / 32; ++w) mm = max(mm, wmax[w]);
+    totals[2] = mm;
+    off[n] = (uint32_t)totals[0];
+  }
 }
 
 cudaError_t launch_cmb_offsets(const uint32_t* cnt_js, int64_t n, uint32_t* off,
@@ -277,23 +288,23 @@ cudaError_t launch_idx16_offsets(const uint32_t* cnt_js, int64_t I, int S, uint3
 }
 
 // ------------------------------------------------------------------------
-// Sparsifier (§3): one CTA selects and compacts the kept channels.
+// Sparsifier (§3): one CTA selects and writes the kept ids and values.
 // ------------------------------------------------------------------------
 constexpr int SPARSIFY_THREADS = 1024;
 
 struct SelLayout {
-  size_t xs, kb, kp, eqw, sel, end;
+  size_t xs, kb, kp, klist, sel, end;
 };
 
-__host__ __device__ inline SelLayout sel_layout(int I, size_t base) {
+__host__ __device__ inline SelLayout sel_layout(int I, size_t base, bool with_list) {
   const size_t nw = (size_t)(I + 31) / 32;
   SelLayout L;
   size_t o = base;
-  L.xs = o;  o += align_up(2 * (size_t)I, 16);
-  L.kb = o;  o += align_up(4 * nw, 16);
-  L.kp = o;  o += align_up(4 * (nw + 1), 16);
-  L.eqw = o; o += align_up(4 * nw, 16);
-  L.sel = o; o += align_up(sizeof(SelShared), 16);
+  L.xs = o;    o += align_up(2 * (size_t)I, 64);   // whole 32-channel words
+  L.kb = o;    o += align_up(4 * nw, 16);
+  L.kp = o;    o += align_up(4 * (nw + 1), 16);
+  L.klist = o; if (with_list) o += align_up(2 * (size_t)I, 16);
+  L.sel = o;   o += align_up(sizeof(SelShared), 16);
   L.end = o;
   return L;
 }
@@ -303,31 +314,20 @@ __global__ void __launch_bounds__(SPARSIFY_THREADS) sparsify_kernel(const uint16
                                                                     uint16_t* __restrict__ kidx,
                                                                     uint16_t* __restrict__ kval) {
   extern __shared__ __align__(128) uint8_t sm[];
-  const SelLayout L = sel_layout(I, 0);
+  const SelLayout L = sel_layout(I, 0, false);
   uint16_t* xs = reinterpret_cast<uint16_t*>(sm + L.xs);
-  uint32_t* kb = reinterpret_cast<uint32_t*>(sm + L.kb);
-  uint32_t* kp = reinterpret_cast<uint32_t*>(sm + L.kp);
-  uint32_t* eqw = reinterpret_cast<uint32_t*>(sm + L.eqw);
   SelShared* sel = reinterpret_cast<SelShared*>(sm + L.sel);
-  load_x_to_smem(xs, x, I);
+  SelKeys K;
+  select_keys_load(K, x, xs, I);
+  select_clear(sel);
   __syncthreads();
-  select_topk(xs, I, k, kb, kp, eqw, sel);
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int nw = (I + 31) >> 5;
-  for (int w = warp; w < nw; w += SPARSIFY_THREADS / 32) {
-    const uint32_t bits = kb[w];
-    if ((bits >> lane) & 1u) {
-      const uint32_t pos = kp[w] + __popc(bits & ((1u << lane) - 1u));
-      const int j = 32 * w + lane;
-      kidx[pos] = (uint16_t)j;
-      kval[pos] = xs[j];
-    }
-  }
+  select_topk(K, xs, I, k, reinterpret_cast<uint32_t*>(sm + L.kb),
+              reinterpret_cast<uint32_t*>(sm + L.kp), kidx, kval, sel);
 }
 
 cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uint16_t* kval,
                             cudaStream_t st) {
-  const size_t smem = sel_layout(I, 0).end;
+  const size_t smem = sel_layout(I, 0, false).end;
   cudaError_t e = cudaFuncSetAttribute(sparsify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
@@ -336,43 +336,49 @@ cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uin
 }
 
 // ------------------------------------------------------------------------
-// spMspV over the bitmask format (§3 product, §4.1 "only the rows ... of
-// non-zero activations are fetched").
+// spMspV over the bitmask format (§3 product; §4.1: only the columns of
+// surviving channels are fetched).
 //
-// Persistent CTAs, one per SM.  The work items are (product p, row segment
-// s, kept index i), ordered p, s, i; CTA b takes the contiguous item range
-// [total*b/G, total*(b+1)/G).  Warp 0 is the producer: its 32 lanes each
-// resolve one item (kept channel id, record offset and size) and issue a
-// 1-D bulk copy of the record into a ring slot in shared memory, signalled
-// on the slot's "full" mbarrier.  Warps 1..NC consume: item v goes to
-// consumer v % NC and slot v % nslot.  A consumer owns, for the current
-// segment, rows 32*lane .. 32*lane+31 in 32 fp32 registers: it reads its
-// mask word, finds where its values start with a warp prefix sum of
-// popcounts, and walks its bits, multiplying each stored fp16 weight by the
-// channel's fp16 activation with an fp32 accumulation.  When a segment ends
-// the consumers add their registers into a shared-memory row tile (rotated
-// so that lanes hit distinct banks) and add the tile to y with vector
-// reductions.
+// Persistent cooperative CTAs, one per SM.  Work items are (product p, row
+// segment s, kept rank i), ordered p, s, i; CTA b takes the contiguous item
+// range [total*b/G, total*(b+1)/G).
 //
-// y is zeroed by the kernel itself: each CTA clears a slice of the outputs
-// at the start and arrives on a split-phase grid barrier; a CTA waits on it
-// only before its first reduction into y, by which time every CTA has long
-// arrived.  The launch is cooperative, so all CTAs are co-resident.
+// Warp 0 produces: lane l resolves items l, l+32, ... (kept channel id,
+// record offset and size; the next PQ-1 items of the lane are resolved ahead
+// so their offset loads are in flight) and issues a 1-D bulk copy of each
+// record into ring slot v % nslot, signalled on the slot's "full" mbarrier
+// with the byte count.  Slots are as large as the largest record of the
+// launch's weights (about 1.3 KB at 50% weight density), so the ring holds
+// as many records as the shared memory allows.
+//
+// Warps 1..NC consume: item v goes to consumer v % NC.  A consumer lane owns
+// rows 32*lane .. 32*lane+31 of the current segment in fp32 registers: it
+// reads its mask word, finds where its values start with a warp prefix sum
+// of popcounts, and walks its bits, multiplying each stored fp16 weight by
+// the channel's fp16 activation (exact product, fp32 accumulation).  When a
+// segment ends the consumers add their registers into a shared-memory row
+// tile (rotated so lanes hit distinct banks) and add the tile to y with
+// vector reductions.
+//
+// y is zeroed by the kernel itself: each CTA clears a slice of the outputs,
+// then arrives on a split-phase grid barrier whose completion it checks only
+// before its first reduction into y.  The launch is cooperative, so all CTAs
+// are co-resident and the barrier cannot deadlock.
 // ------------------------------------------------------------------------
 constexpr int CMB_NC = 16;
 constexpr int CMB_THREADS = 32 * (1 + CMB_NC);
-constexpr int CMB_MAX_SLOTS = 64;
+constexpr int CMB_MAX_SLOTS = 256;
 
 struct CmbLayout {
   SelLayout sel;
   size_t tile, full, empty, meta, ring, total;
 };
 
-__host__ __device__ inline CmbLayout cmb_layout(int I, bool fused, int nslot) {
+__host__ __device__ inline CmbLayout cmb_layout(int I, bool fused, int nslot, int slot_bytes) {
   CmbLayout L;
   size_t o = 0;
   if (fused) {
-    L.sel = sel_layout(I, 0);
+    L.sel = sel_layout(I, 0, true);
     o = L.sel.end;
   }
   L.tile = o;  o += 2 * SEG_ROWS * sizeof(float);
@@ -380,7 +386,7 @@ __host__ __device__ inline CmbLayout cmb_layout(int I, bool fused, int nslot) {
   L.empty = o; o += 8 * (size_t)nslot;
   L.meta = o;  o += align_up(4 * (size_t)nslot, 16);
   o = align_up(o, 128);
-  L.ring = o;  o += (size_t)nslot * MAX_RECORD_BYTES;
+  L.ring = o;  o += (size_t)nslot * slot_bytes;
   L.total = o;
   return L;
 }
@@ -403,20 +409,71 @@ __device__ __forceinline__ void decode_record(const uint8_t* rec, uint16_t xb, f
   }
 }
 
-// Decodes work item u into (product p, segment s, kept index i).
-__device__ __forceinline__ void cmb_item(const CmbArgs& a, int64_t u, int& p, int& s, int& i,
-                                         int64_t& seg_end) {
-  const int64_t k = a.k;
-  int64_t base = 0;
-  p = 0;
-  while (p < a.np - 1 && u >= base + (int64_t)a.p[p].S * k) {
-    base += (int64_t)a.p[p].S * k;
-    ++p;
+// Item cursor: (product p, segment s, kept rank i) of a linear item index.
+struct ItemCursor {
+  int p, s, i;
+  __device__ __forceinline__ void set(const CmbArgs& a, int64_t u) {
+    const int64_t k = a.k;
+    int64_t base = 0;
+    p = 0;
+    while (p < a.np - 1 && u >= base + (int64_t)a.p[p].S * k) {
+      base += (int64_t)a.p[p].S * k;
+      ++p;
+    }
+    const int64_t rem = u - base;
+    s = (int)(rem / k);
+    i = (int)(rem - (int64_t)s * k);
   }
-  const int64_t rem = u - base;
-  s = (int)(rem / k);
-  i = (int)(rem - (int64_t)s * k);
-  seg_end = base + (int64_t)(s + 1) * k;
+  __device__ __forceinline__ void advance(const CmbArgs& a, int n) {
+    i += n;
+    while (i >= a.k) {
+      i -= a.k;
+      if (++s == a.p[p].S) {
+        s = 0;
+        if (p < a.np - 1) ++p;
+      }
+    }
+  }
+};
+
+// Ring position of an item: slot = v % nslot, fill number n = v / nslot.
+struct SlotCursor {
+  int slot, n;
+  __device__ __forceinline__ void set(int v, int nslot) { n = v / nslot; slot = v - n * nslot; }
+  __device__ __forceinline__ void advance(int by, int nslot) {   // by <= nslot
+    slot += by;
+    if (slot >= nslot) { slot -= nslot; ++n; }
+  }
+};
+
+struct Resolved {
+  const uint8_t* src;
+  uint32_t bytes;
+  uint16_t xb;
+  bool bad;
+};
+
+template <bool FUSED>
+__device__ __forceinline__ Resolved resolve_item(const CmbArgs& a, const ItemCursor& c,
+                                                 const uint16_t* klist, const uint16_t* xs) {
+  Resolved r;
+  int j;
+  if (FUSED) {
+    j = klist[c.i];
+    r.xb = xs[j];
+  } else {
+    j = __ldg(a.kidx + c.i);
+    r.xb = __ldg(a.kval + c.i);
+  }
+  r.bad = j >= a.I;
+  if (r.bad) j = 0;   // keep the loads below in bounds; the item is rejected
+  const CmbProb& P = a.p[c.p];
+  const int64_t ri = (int64_t)j * P.S + c.s;
+  const uint32_t o0 = __ldg(P.off + ri), o1 = __ldg(P.off + ri + 1);
+  r.bytes = (o1 - o0) * 16u;
+  r.src = P.data + (size_t)o0 * 16;
+  r.bad = r.bad || o1 < o0 || r.bytes < (uint32_t)MASK_BYTES || r.bytes > (uint32_t)a.slot_bytes;
+  return r;
 }
 
 template <bool FUSED>
@@ -424,28 +481,37 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   extern __shared__ __align__(128) uint8_t sm[];
   __shared__ volatile int abort_flag;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int nslot = a.nslot;
-  const CmbLayout L = cmb_layout(a.I, FUSED, nslot);
+  const int nslot = a.nslot, slot_bytes = a.slot_bytes;
+  const CmbLayout L = cmb_layout(a.I, FUSED, nslot, slot_bytes);
   float* tile = reinterpret_cast<float*>(sm + L.tile);
   uint64_t* full = reinterpret_cast<uint64_t*>(sm + L.full);
   uint64_t* empty = reinterpret_cast<uint64_t*>(sm + L.empty);
   uint32_t* meta = reinterpret_cast<uint32_t*>(sm + L.meta);
   uint8_t* ring = sm + L.ring;
   uint16_t* xs = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.xs) : nullptr;
-  uint32_t* kb = FUSED ? reinterpret_cast<uint32_t*>(sm + L.sel.kb) : nullptr;
-  uint32_t* kp = FUSED ? reinterpret_cast<uint32_t*>(sm + L.sel.kp) : nullptr;
-  const int nw = (a.I + 31) >> 5;
+  uint16_t* klist = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.klist) : nullptr;
+  SelShared* sel = FUSED ? reinterpret_cast<SelShared*>(sm + L.sel.sel) : nullptr;
 
-  if (tid == 0) abort_flag = 0;
+  // ---- prologue: mbarriers, keys of x, tile, this CTA's slice of y = 0 ----
   for (int i = tid; i < nslot; i += CMB_THREADS) {
     mbar_init(&full[i], 1);
     mbar_init(&empty[i], 1);
   }
-  for (int i = tid; i < 2 * SEG_ROWS; i += CMB_THREADS) tile[i] = 0.f;
-  if (FUSED) load_x_to_smem(xs, a.x, a.I);
   fence_mbar_init();
-  __syncthreads();
-  // Zero this CTA's slice of the outputs, then arrive on the grid barrier.
+  SelKeys K;
+  if (FUSED) select_keys_load(K, a.x, xs, a.I);
+  if (tid == 0) {
+    abort_flag = 0;
+    // Warm L2 with this CTA's share of every offset table.
+    for (int p = 0; p < a.np; ++p) {
+      const size_t bytes = align_up(((size_t)a.I * a.p[p].S + 1) * 4, 16);
+      const size_t lo = align_up(bytes * blockIdx.x / gridDim.x, 16);
+      const size_t hi = align_up(bytes * (blockIdx.x + 1) / gridDim.x, 16);
+      if (hi > lo) prefetch_l2(reinterpret_cast<const uint8_t*>(a.p[p].off) + lo, (uint32_t)(hi - lo));
+    }
+  }
+  for (int i = tid; i < 2 * SEG_ROWS; i += CMB_THREADS) tile[i] = 0.f;
+  if (FUSED) select_clear(sel);
   {
     int64_t ytot = 0;
     for (int p = 0; p < a.np; ++p) ytot += a.p[p].O;
@@ -458,105 +524,110 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       base += a.p[p].O;
     }
   }
+  __syncthreads();
   if (FUSED) {
-    select_topk(xs, a.I, a.k, kb, kp, reinterpret_cast<uint32_t*>(sm + L.sel.eqw),
-                reinterpret_cast<SelShared*>(sm + L.sel.sel));
-  } else {
-    __syncthreads();
+    select_topk(K, xs, a.I, a.k, reinterpret_cast<uint32_t*>(sm + L.sel.kb),
+                reinterpret_cast<uint32_t*>(sm + L.sel.kp), klist, nullptr, sel);
   }
-  __shared__ unsigned int bar_gen0;
-  if (tid == 0) {
-    __threadfence();
-    bar_gen0 = ld_acquire_gpu(a.bar + 1);
-    if (atomicAdd(a.bar, 1u) == gridDim.x - 1) {
-      a.bar[0] = 0u;
-      __threadfence();
-      atomicAdd(a.bar + 1, 1u);
-    }
-  }
-  __syncthreads();   // publishes bar_gen0
 
-  const int64_t k = a.k;
   int64_t total = 0;
-  for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * k;
+  for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
   const int64_t u0 = total * blockIdx.x / gridDim.x;
   const int64_t u1 = total * (blockIdx.x + 1) / gridDim.x;
-  const int64_t nv = u1 - u0;
+  const int nv = (int)(u1 - u0);
 
   if (warp == 0) {
     // ---------------- producer ----------------
+    constexpr int PQ = 4;
     const uint64_t pol = policy_evict_first();
-    int64_t last_v = -1;
-    for (int64_t vb = 0; vb < nv; vb += 32) {
-      if (abort_flag) break;
-      const int64_t v = vb + lane;
-      if (v >= nv) continue;
-      int p, s, i;
-      int64_t seg_end;
-      cmb_item(a, u0 + v, p, s, i, seg_end);
-      int j;
-      uint16_t xb;
-      if (FUSED) {
-        j = kept_channel(kb, kp, nw, (uint32_t)i);
-        xb = xs[j];
-      } else {
-        j = __ldg(a.kidx + i);
-        xb = __ldg(a.kval + i);
+    int last_v = -1;
+    bool stop = false;
+    ItemCursor cur;
+    cur.set(a, u0 + lane);
+    SlotCursor sc;
+    sc.set(lane, nslot);
+    Resolved q[PQ];
+#pragma unroll
+    for (int d = 0; d < PQ; ++d) {
+      if (lane + 32 * d < nv) {
+        if (d > 0) cur.advance(a, 32);
+        q[d] = resolve_item<FUSED>(a, cur, klist, xs);
       }
-      if (j < 0 || j >= a.I) {
-        atomicOr(&g_status, STATUS_FORMAT);
-        abort_flag = 1;
-        break;
+    }
+    for (int v0 = lane; v0 < nv && !stop; v0 += 32 * PQ) {
+#pragma unroll
+      for (int d = 0; d < PQ; ++d) {
+        const int v = v0 + 32 * d;
+        if (stop || v >= nv) continue;
+        if (abort_flag) { stop = true; continue; }
+        const Resolved r = q[d];
+        if (r.bad) {
+          atomicOr(&g_status, STATUS_FORMAT);
+          abort_flag = 1;
+          stop = true;
+          continue;
+        }
+        if (v + 32 * PQ < nv) {                 // refill: this lane's item v + 32*PQ
+          cur.advance(a, 32);
+          q[d] = resolve_item<FUSED>(a, cur, klist, xs);
+        }
+        if (sc.n > 0 && !mbar_wait_bounded(&empty[sc.slot], (uint32_t)((sc.n - 1) & 1), &abort_flag)) {
+          stop = true;
+          continue;
+        }
+        meta[sc.slot] = r.xb;
+        mbar_arrive_expect_tx(&full[sc.slot], r.bytes);
+        bulk_g2s(ring + (size_t)sc.slot * slot_bytes, r.src, r.bytes, &full[sc.slot], pol);
+        last_v = v;
+        sc.advance(32, nslot);
       }
-      const CmbProb& P = a.p[p];
-      const int64_t ri = (int64_t)j * P.S + s;
-      const uint32_t o0 = __ldg(P.off + ri), o1 = __ldg(P.off + ri + 1);
-      const uint32_t bytes = (o1 - o0) * 16u;
-      if (o1 < o0 || bytes < (uint32_t)MASK_BYTES || bytes > (uint32_t)MAX_RECORD_BYTES) {
-        atomicOr(&g_status, STATUS_FORMAT);
-        abort_flag = 1;
-        break;
-      }
-      const int slot = (int)(v % nslot);
-      const int64_t n = v / nslot;
-      if (n > 0 && !mbar_wait_bounded(&empty[slot], (uint32_t)((n - 1) & 1), &abort_flag)) break;
-      meta[slot] = xb;
-      mbar_arrive_expect_tx(&full[slot], bytes);
-      bulk_g2s(ring + (size_t)slot * MAX_RECORD_BYTES, P.data + (size_t)o0 * 16, bytes, &full[slot],
-               pol);
-      last_v = v;
     }
     if (abort_flag) {
       // Let this lane's copies still in flight land before the CTA exits.
-      for (int64_t v = last_v; v >= 0 && v > last_v - nslot; v -= 32)
-        mbar_wait_limited(&full[v % nslot], (uint32_t)((v / nslot) & 1));
+      for (int v = last_v; v >= 0 && v > last_v - nslot; v -= 32) {
+        SlotCursor w;
+        w.set(v, nslot);
+        mbar_wait_limited(&full[w.slot], (uint32_t)(w.n & 1));
+      }
     }
   } else {
     // ---------------- consumers ----------------
     const int c = warp - 1;
     const int ctid = tid - 32;
+    // Arrive on the grid barrier once this CTA's slice of y is zero (ordered
+    // by the __syncthreads above); done here, off the selection's path, its
+    // latency overlaps the first record fetches.
+    unsigned int gen0 = 0;
+    if (ctid == 0) {
+      gen0 = ld_relaxed_gpu(a.bar + 1);
+      if (atom_add_acq_rel_gpu(a.bar, 1u) == gridDim.x - 1) {   // last arriver opens it
+        a.bar[0] = 0u;
+        red_add_release_gpu(a.bar + 1, 1u);
+      }
+    }
     float acc[32];
     int64_t u = u0;
     int piece = 0;
     while (u < u1) {
-      int p, s, i0;
-      int64_t seg_end;
-      cmb_item(a, u, p, s, i0, seg_end);
+      ItemCursor pc;
+      pc.set(a, u);
+      const int64_t seg_end = u + (a.k - pc.i);   // end of this (p, s) run
       const int64_t pend = seg_end < u1 ? seg_end : u1;
-      const int64_t va = u - u0, vb = pend - u0;
+      const int va = (int)(u - u0), vb = (int)(pend - u0);
 #pragma unroll
       for (int t = 0; t < 32; ++t) acc[t] = 0.f;
       bool any = false;
-      int64_t v = va + ((c - (int)(va % CMB_NC)) % CMB_NC + CMB_NC) % CMB_NC;
+      int v = va + ((c - va % CMB_NC) % CMB_NC + CMB_NC) % CMB_NC;
+      SlotCursor sc;
+      sc.set(v, nslot);
       for (; v < vb; v += CMB_NC) {
-        const int slot = (int)(v % nslot);
-        const uint32_t par = (uint32_t)((v / nslot) & 1);
-        if (!abort_flag && mbar_wait_bounded(&full[slot], par, &abort_flag)) {
-          decode_record(ring + (size_t)slot * MAX_RECORD_BYTES, (uint16_t)meta[slot], acc, lane);
+        if (!abort_flag && mbar_wait_bounded(&full[sc.slot], (uint32_t)(sc.n & 1), &abort_flag)) {
+          decode_record(ring + (size_t)sc.slot * slot_bytes, (uint16_t)meta[sc.slot], acc, lane);
           any = true;
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[slot]);
+        if (lane == 0) mbar_arrive(&empty[sc.slot]);
+        sc.advance(CMB_NC, nslot);
       }
       float* tb = tile + (piece & 1) * SEG_ROWS;
       if (any) {
@@ -566,7 +637,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       if (piece == 0 && ctid == 0) {
         // First reduction into y: every CTA must have zeroed its slice.
         const uint64_t t0 = globaltimer_ns();
-        while (ld_acquire_gpu(a.bar + 1) == bar_gen0) {
+        while (ld_acquire_gpu(a.bar + 1) == gen0) {
           if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
             atomicOr(&g_status, STATUS_TIMEOUT);
             abort_flag = 1;
@@ -575,9 +646,9 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
         }
       }
       named_bar_sync(1, CMB_NC * 32);
-      const CmbProb& P = a.p[p];
-      const int rows = min(SEG_ROWS, P.O - s * SEG_ROWS);
-      float* yb = P.y + (size_t)s * SEG_ROWS;
+      const CmbProb& P = a.p[pc.p];
+      const int rows = min(SEG_ROWS, P.O - pc.s * SEG_ROWS);
+      float* yb = P.y + (size_t)pc.s * SEG_ROWS;
       for (int g = ctid; 4 * g < rows; g += CMB_NC * 32) {
         float vv[4];
 #pragma unroll
@@ -609,18 +680,24 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   cudaError_t e = dev_props(&dp);
   if (e != cudaSuccess) return e;
   const bool fused = a.kidx == nullptr;
-  const size_t fixed = cmb_layout(a.I, fused, 0).total + 256;
-  const size_t per_slot = MAX_RECORD_BYTES + 8 + 8 + 4;
-  int nslot = 0;
-  if ((size_t)dp.smem_optin > fixed) nslot = (int)(((size_t)dp.smem_optin - fixed) / per_slot);
-  nslot = std::min(nslot, CMB_MAX_SLOTS) / CMB_NC * CMB_NC;
-  if (nslot < 32) return cudaErrorInvalidValue;
-  a.nslot = nslot;
-  const size_t smem = cmb_layout(a.I, fused, nslot).total;
   int64_t total = 0;
   for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
   if (total <= 0) return cudaSuccess;
   const int grid = (int)std::min<int64_t>(dp.nsm, total);
+  if ((total + grid - 1) / grid >= (int64_t)1 << 30) return cudaErrorInvalidValue;
+  // Slot size: the largest record among the launch's weights (given by the
+  // caller in a.slot_bytes); slot count: as many as the shared memory holds.
+  const int slot_bytes = (int)align_up((size_t)std::max(a.slot_bytes, MASK_BYTES + 16), 16);
+  if (slot_bytes > MAX_RECORD_BYTES) return cudaErrorInvalidValue;
+  const size_t avail = (size_t)dp.smem_optin - 256;   // static shared memory headroom
+  const size_t fixed = cmb_layout(a.I, fused, 0, slot_bytes).total + 128;
+  if (fixed >= avail) return cudaErrorInvalidValue;
+  int nslot = (int)((avail - fixed) / (slot_bytes + 20));
+  nslot = std::min(nslot, CMB_MAX_SLOTS);
+  if (nslot < 32) return cudaErrorInvalidValue;
+  a.nslot = nslot;
+  a.slot_bytes = slot_bytes;
+  const size_t smem = cmb_layout(a.I, fused, nslot, slot_bytes).total;
   void (*kern)(const CmbArgs) = fused ? cmb_spmspv_kernel<true> : cmb_spmspv_kernel<false>;
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
@@ -643,29 +720,30 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
 // spMspV over the index format (parity format): one warp per kept channel,
 // lanes stride its non-zeros and add w * x into y[row] atomically.
 // ------------------------------------------------------------------------
-constexpr int IDX16_THREADS = 256;
+constexpr int IDX16_THREADS = 512;   // the selection needs >= 512 threads
 
 template <bool FUSED>
 __global__ void __launch_bounds__(IDX16_THREADS) idx16_spmspv_kernel(const Idx16Args a) {
   extern __shared__ __align__(128) uint8_t sm[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int nw = (a.I + 31) >> 5;
-  const SelLayout L = sel_layout(a.I, 0);
+  const SelLayout L = sel_layout(a.I, 0, true);
   uint16_t* xs = reinterpret_cast<uint16_t*>(sm + L.xs);
-  uint32_t* kb = reinterpret_cast<uint32_t*>(sm + L.kb);
-  uint32_t* kp = reinterpret_cast<uint32_t*>(sm + L.kp);
+  uint16_t* klist = reinterpret_cast<uint16_t*>(sm + L.klist);
   if (FUSED) {
-    load_x_to_smem(xs, a.x, a.I);
+    SelShared* sel = reinterpret_cast<SelShared*>(sm + L.sel);
+    SelKeys K;
+    select_keys_load(K, a.x, xs, a.I);
+    select_clear(sel);
     __syncthreads();
-    select_topk(xs, a.I, a.k, kb, kp, reinterpret_cast<uint32_t*>(sm + L.eqw),
-                reinterpret_cast<SelShared*>(sm + L.sel));
+    select_topk(K, xs, a.I, a.k, reinterpret_cast<uint32_t*>(sm + L.kb),
+                reinterpret_cast<uint32_t*>(sm + L.kp), klist, nullptr, sel);
   }
   const int nwt = gridDim.x * (IDX16_THREADS / 32);
   for (int i = blockIdx.x * (IDX16_THREADS / 32) + warp; i < a.k; i += nwt) {
     int j;
     uint16_t xb;
     if (FUSED) {
-      j = kept_channel(kb, kp, nw, (uint32_t)i);
+      j = klist[i];
       xb = xs[j];
     } else {
       j = __ldg(a.kidx + i);
@@ -692,7 +770,7 @@ cudaError_t launch_idx16_spmspv(const Idx16Args& a, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   if (a.k <= 0) return cudaSuccess;
   const bool fused = a.kidx == nullptr;
-  const size_t smem = fused ? sel_layout(a.I, 0).end : 0;
+  const size_t smem = fused ? sel_layout(a.I, 0, true).end : 0;
   const int warps = IDX16_THREADS / 32;
   const int grid = (int)std::min<int64_t>((int64_t)dp.nsm * 2, ((int64_t)a.k + warps - 1) / warps);
   if (fused) {
