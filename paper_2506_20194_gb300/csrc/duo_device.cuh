@@ -218,88 +218,49 @@ __device__ inline void load_x_to_smem(uint16_t* xs, const uint16_t* x, int I) {
   }
 }
 
-constexpr int SEL_BINS = 4096;   // histogram of key >> 3
+constexpr int SEL_BINS = 2048;   // histogram of key >> 4
 
 // Shared state of the selection.
 struct SelShared {
   uint32_t hist[SEL_BINS];
+  uint32_t sub[16];      // key & 15 inside the threshold bin
   uint32_t wtot[32];     // per-warp partial sums
-  uint32_t sub[32][4];   // per-warp counts of key & 7 inside the threshold bin (16-bit pairs)
-  uint32_t B;            // threshold bin
-  uint32_t aboveB;       // channels in bins above it
+  uint32_t C;            // threshold bin
+  uint32_t aboveC;       // channels in bins above it
 };
 
-// Clears the histogram (before the __syncthreads that precedes select_topk).
+// Clears the histograms (before the __syncthreads that precedes select_topk).
 __device__ __forceinline__ void select_clear(SelShared* sh) {
   uint4* h = reinterpret_cast<uint4*>(sh->hist);
   for (int i = threadIdx.x; i < SEL_BINS / 4; i += blockDim.x) h[i] = make_uint4(0u, 0u, 0u, 0u);
+  if (threadIdx.x < 16) sh->sub[threadIdx.x] = 0u;
 }
 
 // Exact top-k by magnitude (§3): keeps the k channels with the largest
 // |x_j|, ties to the lower index.  The key of x_j is its fp16 bit pattern
 // with the sign cleared; for IEEE fp16 this integer order equals the order of
-// |x_j| (NaN patterns sort above Inf).
+// |x_j| (NaN patterns sort above Inf).  xs holds the fp16 bits of x in
+// shared memory (room for a whole number of 32-channel words).
 //
-//  1. histogram of key >> 3 (4096 bins, shared-memory atomics; a thread's
-//     keys are in registers);
-//  2. suffix scan of the histogram (512 threads x 8 bins) to find the bin B
+//  1. histogram of key >> 4 (2048 bins, shared-memory atomics);
+//  2. suffix scan of the histogram (512 threads x 4 bins) to find the bin C
 //     where the count from the top reaches k;
-//  3. per-warp counts of the 8 keys inside bin B (warp reductions, no
-//     atomics) give the threshold key T and the count above it; the
-//     q = k - count(key > T) lowest-indexed channels with key == T are kept;
+//  3. histogram of key & 15 over the few channels in bin C, giving the
+//     threshold key T and the count above it; the q = k - count(key > T)
+//     lowest-indexed channels with key == T are kept;
 //  4. every thread builds the "above T" / "equal to T" masks of its own
 //     32-channel words from 16-byte loads of x, a block exclusive scan of the
 //     packed counts orders the words, and the thread writes kb[w] (kept
 //     bitmap, bit b <-> channel 32w+b) and kp[w] (kept channels before word
 //     w; kp[nw] = k);
-//  5. warps emit klist[r] (channel of kept rank r, ascending) and kvals[r]
-//     (its fp16 bits) word by word, lane = bit, if requested.
-// Shared-memory accesses are arranged to be bank-conflict free (rotated
-// 16-byte chunks).
+//  5. if klist / kvals are given, warps emit klist[r] (channel of kept rank
+//     r, ascending) and kvals[r] (its fp16 bits), lane = bit.
+// Shared-memory accesses are arranged to be bank-conflict free.
 //
-// select_keys_load() runs first (it also writes xs, the fp16 bits of x, to
-// shared memory; xs needs room for a multiple of 32 entries), then
-// select_clear(), then a __syncthreads.  All threads of the block take part
-// (blockDim.x >= 512, a multiple of 32); it ends with a __syncthreads.
-constexpr int SEL_MAXKEYS = 32;   // keys per thread kept in registers
-constexpr uint32_t KEY_NONE = 0xFFFFu;
-
-struct SelKeys {
-  uint32_t key[SEL_MAXKEYS];
-  int n;   // keys held (channels tid, tid + blockDim, ...)
-};
-
-__device__ __forceinline__ void select_keys_load(SelKeys& K, const uint16_t* __restrict__ x,
-                                                 uint16_t* xs, int I) {
-  const int nt = blockDim.x;
-  K.n = (I - (int)threadIdx.x + nt - 1) / nt;
-  if (K.n <= SEL_MAXKEYS) {
-#pragma unroll
-    for (int r = 0; r < SEL_MAXKEYS; ++r) {
-      const int j = threadIdx.x + r * nt;
-      uint32_t v = KEY_NONE;
-      if (j < I) {
-        const uint16_t b = x[j];
-        xs[j] = b;
-        v = b & 0x7FFFu;
-      }
-      K.key[r] = v;
-    }
-  } else {
-    load_x_to_smem(xs, x, I);
-  }
-}
-
-template <typename F>
-__device__ __forceinline__ void for_each_key(const SelKeys& K, const uint16_t* xs, int I, F f) {
-  if (K.n <= SEL_MAXKEYS) {
-#pragma unroll
-    for (int r = 0; r < SEL_MAXKEYS; ++r)
-      if (K.key[r] != KEY_NONE) f(K.key[r]);
-  } else {
-    for (int j = threadIdx.x; j < I; j += blockDim.x) f((uint32_t)(xs[j] & 0x7FFFu));
-  }
-}
+// select_clear() and the loading of xs come first, then a __syncthreads.
+// All threads of the block take part (blockDim.x >= 512, a multiple of 32);
+// it ends with a __syncthreads.
+__device__ __forceinline__ uint32_t key_of(const uint16_t* xs, int j) { return xs[j] & 0x7FFFu; }
 
 // Masks of the channels of word w (32 channels) above T and equal to T.  The
 // four 16-byte chunks are read in an order rotated by (w >> 1) so that the
@@ -331,8 +292,8 @@ __device__ __forceinline__ void word_masks(const uint16_t* xs, int I, int w, boo
   eq &= vmask;
 }
 
-__device__ inline void select_topk(const SelKeys& K, const uint16_t* xs, int I, int k, uint32_t* kb,
-                                   uint32_t* kp, uint16_t* klist, uint16_t* kvals, SelShared* sh) {
+__device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t* kb, uint32_t* kp,
+                                   uint16_t* klist, uint16_t* kvals, SelShared* sh) {
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, wid = tid >> 5;
   const int nwarps = nt >> 5;
   const int nw = (I + 31) >> 5;
@@ -340,20 +301,26 @@ __device__ inline void select_topk(const SelKeys& K, const uint16_t* xs, int I, 
   uint32_t T = 0u;
   int q = 0;
   if (!all && !none) {
-    // 1. histogram of the high 12 key bits
-    for_each_key(K, xs, I, [&](uint32_t key) { atomicAdd(&sh->hist[key >> 3], 1u); });
+    // 1. histogram of the high 11 key bits
+    {
+      int j = tid;
+      for (; j + 3 * nt < I; j += 4 * nt) {
+        const uint32_t k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
+        const uint32_t k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
+        atomicAdd(&sh->hist[k0 >> 4], 1u);
+        atomicAdd(&sh->hist[k1 >> 4], 1u);
+        atomicAdd(&sh->hist[k2 >> 4], 1u);
+        atomicAdd(&sh->hist[k3 >> 4], 1u);
+      }
+      for (; j < I; j += nt) atomicAdd(&sh->hist[key_of(xs, j) >> 4], 1u);
+    }
     __syncthreads();
-    // 2. suffix scan: thread t < 512 owns bins [8t, 8t + 8)
-    uint32_t c[8], s = 0, incl = 0;
+    // 2. suffix scan: thread t < 512 owns bins [4t, 4t + 4)
+    uint32_t c[4] = {0u, 0u, 0u, 0u}, s = 0, incl = 0;
     if (tid < 512) {
-      const uint4* hp = reinterpret_cast<const uint4*>(sh->hist) + 2 * tid;
-      const int r = (tid >> 2) & 1;   // rotated halves: conflict-free quarter warps
-      const uint4 ha = hp[r], hb = hp[r ^ 1];
-      const uint4 h0 = r ? hb : ha, h1 = r ? ha : hb;
-      c[0] = h0.x; c[1] = h0.y; c[2] = h0.z; c[3] = h0.w;
-      c[4] = h1.x; c[5] = h1.y; c[6] = h1.z; c[7] = h1.w;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) s += c[i];
+      const uint4 h = reinterpret_cast<const uint4*>(sh->hist)[tid];
+      c[0] = h.x; c[1] = h.y; c[2] = h.z; c[3] = h.w;
+      s = c[0] + c[1] + c[2] + c[3];
       incl = s;   // suffix over lanes >= lane inside the warp
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
@@ -366,59 +333,45 @@ __device__ inline void select_topk(const SelKeys& K, const uint16_t* xs, int I, 
     if (tid < 512) {
       uint32_t above_w = (lane > wid && lane < 16) ? sh->wtot[lane] : 0u;
       above_w = __reduce_add_sync(FULL_MASK, above_w);
-      const uint32_t hi = above_w + incl;   // channels in bins >= 8*tid
-      const uint32_t lo = hi - s;           // channels in bins >= 8*tid + 8
+      const uint32_t hi = above_w + incl;   // channels in bins >= 4*tid
+      const uint32_t lo = hi - s;           // channels in bins >= 4*tid + 4
       if (lo < (uint32_t)k && (uint32_t)k <= hi) {
         uint32_t acc = lo;
         int b = 0;
 #pragma unroll
-        for (int i = 7; i >= 0; --i) {
+        for (int i = 3; i >= 0; --i) {
           if (acc + c[i] >= (uint32_t)k) { b = i; break; }
           acc += c[i];
         }
-        sh->B = 8u * tid + (uint32_t)b;
-        sh->aboveB = acc;
+        sh->C = 4u * tid + (uint32_t)b;
+        sh->aboveC = acc;
       }
     }
     __syncthreads();
-    // 3. the 8 keys of bin B: per-thread counts in 16-bit fields, reduced
-    //    per warp, then summed over warps
-    const uint32_t B = sh->B;
-    uint32_t cnt[4] = {0u, 0u, 0u, 0u};
-    for_each_key(K, xs, I, [&](uint32_t key) {
-      if ((key >> 3) == B) {
-        const uint32_t low = key & 7u;
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          cnt[v] += (low == 2u * v) ? 1u : 0u;
-          cnt[v] += (low == 2u * v + 1u) ? 0x10000u : 0u;
-        }
-      }
-    });
-#pragma unroll
-    for (int v = 0; v < 4; ++v) cnt[v] = __reduce_add_sync(FULL_MASK, cnt[v]);
-    if (lane == 0) {
-#pragma unroll
-      for (int v = 0; v < 4; ++v) sh->sub[wid][v] = cnt[v];
+    // 3. the 16 keys of bin C (few channels: contention-free atomics)
+    const uint32_t C = sh->C;
+    for (int j = tid; j < I; j += nt) {
+      const uint32_t key = key_of(xs, j);
+      if ((key >> 4) == C) atomicAdd(&sh->sub[key & 15u], 1u);
     }
     __syncthreads();
-    uint32_t tot4[4] = {0u, 0u, 0u, 0u};
-    for (int w2 = 0; w2 < nwarps; ++w2) {
+    uint32_t sub[16];
 #pragma unroll
-      for (int v = 0; v < 4; ++v) tot4[v] += sh->sub[w2][v];
+    for (int i = 0; i < 4; ++i) {
+      const uint4 v = reinterpret_cast<const uint4*>(sh->sub)[i];
+      sub[4 * i] = v.x; sub[4 * i + 1] = v.y; sub[4 * i + 2] = v.z; sub[4 * i + 3] = v.w;
     }
-    uint32_t above = sh->aboveB;
+    uint32_t above = sh->aboveC;
     int b = -1;
 #pragma unroll
-    for (int v = 7; v >= 0; --v) {
-      const uint32_t cv = (tot4[v >> 1] >> (16 * (v & 1))) & 0xFFFFu;
+    for (int v = 15; v >= 0; --v) {
       if (b < 0) {
-        if (above + cv >= (uint32_t)k) b = v;
-        else above += cv;
+        if (above + sub[v] >= (uint32_t)k) b = v;
+        else above += sub[v];
       }
     }
     if (b < 0) b = 0;
-    T = 8u * B + (uint32_t)b;
+    T = 16u * C + (uint32_t)b;
     q = k - (int)above;
   }
   // 4. thread tid owns words [w0, w1)
@@ -433,8 +386,7 @@ __device__ inline void select_topk(const SelKeys& K, const uint16_t* xs, int I, 
     packed += (uint32_t)__popc(gt) | ((uint32_t)__popc(eq) << 16);
   }
   const uint32_t inc = warp_inclusive_scan(packed, lane);
-  __syncthreads();   // wtot of step 2 is no longer read
-  if (lane == 31) sh->wtot[wid] = inc;
+  if (lane == 31) sh->wtot[wid] = inc;   // step 2's wtot reads ended two barriers ago
   __syncthreads();
   if (wid == 0) {
     uint32_t t = lane < nwarps ? sh->wtot[lane] : 0u;

@@ -317,11 +317,10 @@ __global__ void __launch_bounds__(SPARSIFY_THREADS) sparsify_kernel(const uint16
   const SelLayout L = sel_layout(I, 0, false);
   uint16_t* xs = reinterpret_cast<uint16_t*>(sm + L.xs);
   SelShared* sel = reinterpret_cast<SelShared*>(sm + L.sel);
-  SelKeys K;
-  select_keys_load(K, x, xs, I);
+  load_x_to_smem(xs, x, I);
   select_clear(sel);
   __syncthreads();
-  select_topk(K, xs, I, k, reinterpret_cast<uint32_t*>(sm + L.kb),
+  select_topk(xs, I, k, reinterpret_cast<uint32_t*>(sm + L.kb),
               reinterpret_cast<uint32_t*>(sm + L.kp), kidx, kval, sel);
 }
 
@@ -392,6 +391,30 @@ __host__ __device__ inline CmbLayout cmb_layout(int I, bool fused, int nslot, in
 }
 
 __device__ __forceinline__ int tile_index(int r) { return (r & ~31) | ((r + (r >> 5)) & 31); }
+
+// One consumer warp decodes two records of the same segment at once: one
+// warp prefix sum serves both masks (16-bit halves) and the two records'
+// loads interleave.  Lane owns rows 32*lane + t.
+__device__ __forceinline__ void decode_two(const uint8_t* ra, uint16_t xa, const uint8_t* rb,
+                                           uint16_t xb, float (&acc)[32], int lane) {
+  const uint32_t ma = reinterpret_cast<const uint32_t*>(ra)[lane];
+  const uint32_t mb = reinterpret_cast<const uint32_t*>(rb)[lane];
+  const uint32_t c = (uint32_t)__popc(ma) | ((uint32_t)__popc(mb) << 16);
+  const uint32_t ex = warp_inclusive_scan(c, lane) - c;
+  const uint16_t* pa = reinterpret_cast<const uint16_t*>(ra + MASK_BYTES) + (ex & 0xFFFFu);
+  const uint16_t* pb = reinterpret_cast<const uint16_t*>(rb + MASK_BYTES) + (ex >> 16);
+#pragma unroll
+  for (int t = 0; t < 32; ++t) {
+    if (ma & (1u << t)) {
+      acc[t] = fma_f16_f32(*pa, xa, acc[t]);
+      ++pa;
+    }
+    if (mb & (1u << t)) {
+      acc[t] = fma_f16_f32(*pb, xb, acc[t]);
+      ++pb;
+    }
+  }
+}
 
 // One consumer warp decodes one record: lane owns rows 32*lane + t.
 __device__ __forceinline__ void decode_record(const uint8_t* rec, uint16_t xb, float (&acc)[32],
@@ -489,17 +512,18 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   uint32_t* meta = reinterpret_cast<uint32_t*>(sm + L.meta);
   uint8_t* ring = sm + L.ring;
   uint16_t* xs = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.xs) : nullptr;
+  uint32_t* kb = FUSED ? reinterpret_cast<uint32_t*>(sm + L.sel.kb) : nullptr;
+  uint32_t* kp = FUSED ? reinterpret_cast<uint32_t*>(sm + L.sel.kp) : nullptr;
   uint16_t* klist = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.klist) : nullptr;
   SelShared* sel = FUSED ? reinterpret_cast<SelShared*>(sm + L.sel.sel) : nullptr;
 
-  // ---- prologue: mbarriers, keys of x, tile, this CTA's slice of y = 0 ----
+  // ---- prologue: x, mbarriers, tile, this CTA's slice of y = 0 ----
+  if (FUSED) load_x_to_smem(xs, a.x, a.I);   // issued first: its latency overlaps the rest
   for (int i = tid; i < nslot; i += CMB_THREADS) {
     mbar_init(&full[i], 1);
     mbar_init(&empty[i], 1);
   }
   fence_mbar_init();
-  SelKeys K;
-  if (FUSED) select_keys_load(K, a.x, xs, a.I);
   if (tid == 0) {
     abort_flag = 0;
     // Warm L2 with this CTA's share of every offset table.
@@ -525,10 +549,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     }
   }
   __syncthreads();
-  if (FUSED) {
-    select_topk(K, xs, a.I, a.k, reinterpret_cast<uint32_t*>(sm + L.sel.kb),
-                reinterpret_cast<uint32_t*>(sm + L.sel.kp), klist, nullptr, sel);
-  }
+  if (FUSED) select_topk(xs, a.I, a.k, kb, kp, klist, nullptr, sel);
 
   int64_t total = 0;
   for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
@@ -618,16 +639,31 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       for (int t = 0; t < 32; ++t) acc[t] = 0.f;
       bool any = false;
       int v = va + ((c - va % CMB_NC) % CMB_NC + CMB_NC) % CMB_NC;
-      SlotCursor sc;
+      SlotCursor sc, sc2;
       sc.set(v, nslot);
-      for (; v < vb; v += CMB_NC) {
+      sc2.set(v + CMB_NC, nslot);
+      for (; v + CMB_NC < vb; v += 2 * CMB_NC) {   // this consumer's items in pairs
+        if (!abort_flag && mbar_wait_bounded(&full[sc.slot], (uint32_t)(sc.n & 1), &abort_flag) &&
+            mbar_wait_bounded(&full[sc2.slot], (uint32_t)(sc2.n & 1), &abort_flag)) {
+          decode_two(ring + (size_t)sc.slot * slot_bytes, (uint16_t)meta[sc.slot],
+                     ring + (size_t)sc2.slot * slot_bytes, (uint16_t)meta[sc2.slot], acc, lane);
+          any = true;
+        }
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&empty[sc.slot]);
+          mbar_arrive(&empty[sc2.slot]);
+        }
+        sc.advance(2 * CMB_NC, nslot);
+        sc2.advance(2 * CMB_NC, nslot);
+      }
+      if (v < vb) {
         if (!abort_flag && mbar_wait_bounded(&full[sc.slot], (uint32_t)(sc.n & 1), &abort_flag)) {
           decode_record(ring + (size_t)sc.slot * slot_bytes, (uint16_t)meta[sc.slot], acc, lane);
           any = true;
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[sc.slot]);
-        sc.advance(CMB_NC, nslot);
       }
       float* tb = tile + (piece & 1) * SEG_ROWS;
       if (any) {
@@ -723,7 +759,7 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
 constexpr int IDX16_THREADS = 512;   // the selection needs >= 512 threads
 
 template <bool FUSED>
-__global__ void __launch_bounds__(IDX16_THREADS) idx16_spmspv_kernel(const Idx16Args a) {
+__global__ void __launch_bounds__(IDX16_THREADS, 1) idx16_spmspv_kernel(const Idx16Args a) {
   extern __shared__ __align__(128) uint8_t sm[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const SelLayout L = sel_layout(a.I, 0, true);
@@ -731,11 +767,10 @@ __global__ void __launch_bounds__(IDX16_THREADS) idx16_spmspv_kernel(const Idx16
   uint16_t* klist = reinterpret_cast<uint16_t*>(sm + L.klist);
   if (FUSED) {
     SelShared* sel = reinterpret_cast<SelShared*>(sm + L.sel);
-    SelKeys K;
-    select_keys_load(K, a.x, xs, a.I);
+    load_x_to_smem(xs, a.x, a.I);
     select_clear(sel);
     __syncthreads();
-    select_topk(K, xs, a.I, a.k, reinterpret_cast<uint32_t*>(sm + L.kb),
+    select_topk(xs, a.I, a.k, reinterpret_cast<uint32_t*>(sm + L.kb),
                 reinterpret_cast<uint32_t*>(sm + L.kp), klist, nullptr, sel);
   }
   const int nwt = gridDim.x * (IDX16_THREADS / 32);
