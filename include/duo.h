@@ -171,6 +171,44 @@ int duo_packed_query(const duo_packed* h, duo_packed_info* info);
  * Errors: DUO_EINVAL (dead handle, which, NULL dst, size mismatch), DUO_ECUDA. */
 int duo_packed_export(const duo_packed* h, int which, void* dst_host, int64_t bytes);
 
+/*
+ * duo_pack_cmb_noalloc -- the bitmask packing of duo_pack (same bytes)
+ * without any device allocation.  The paper has no counterpart: this entry
+ * point exists for callers that cannot call cudaMalloc themselves, such as
+ * an engine that hands out all device memory from its own pool, or a
+ * process whose device allocations someone else accounts for.  duo_pack
+ * needs per-record scratch and allocates it (and the packed buffers); this
+ * variant writes into buffers the caller provides and keeps its scratch in a
+ * fixed file-scope device array of the library.
+ *
+ *   W_fp16_dev, out, in, ldw : as in duo_pack.
+ *   off_dev       : device, uint32[in * ceil(out/1024) + 1], 4-byte aligned:
+ *                   receives the record offsets (16-byte units).
+ *   data_dev      : device, 16-byte aligned, data_capacity bytes: receives
+ *                   the records.  NULL asks only for the size.
+ *   data_bytes    : host out: the packed data size in bytes.
+ *   stream        : work is enqueued on it; the call synchronises it.
+ *
+ * Limits and behaviour:
+ *   - in * ceil(out/1024) must not exceed DUO_NOALLOC_MAX_RECORDS (the
+ *     scratch holds one 32-bit count per record), else DUO_ERANGE;
+ *   - data_capacity smaller than the packed size: DUO_ERANGE, with
+ *     *data_bytes set to the size needed;
+ *   - calls no cudaMalloc, cudaFree or other allocating routine;
+ *   - the scratch array (about 1 MiB) is held by every GPU that loads the
+ *     library until the process exits; every call shares it and the previous
+ *     call's contents are never read, but calls that overlap on the GPU
+ *     (concurrent calls from several threads or streams) race on it;
+ *   - the first call on a device looks up the array's device address with
+ *     that device current; make that first call before any stream capture
+ *     (the call synchronises its stream and cannot be captured anyway).
+ * Errors: DUO_EINVAL, DUO_ERANGE, DUO_ECUDA.
+ */
+#define DUO_NOALLOC_MAX_RECORDS 262144
+int duo_pack_cmb_noalloc(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw,
+                         uint32_t* off_dev, void* data_dev, int64_t data_capacity,
+                         int64_t* data_bytes, void* stream);
+
 /* Synchronises `stream`, returns and clears the device status word:
  * DUO_OK; DUO_ETIMEOUT if a bounded device wait ran out since the last
  * call; DUO_EFORMAT if a kernel met a record size or channel id outside the

@@ -55,11 +55,13 @@ def load_library(path: str | None = None):
     lib.duo_free.argtypes = [vp]
     lib.duo_packed_query.argtypes = [vp, ctypes.POINTER(_Info)]
     lib.duo_packed_export.argtypes = [vp, i32, vp, i64]
+    lib.duo_pack_cmb_noalloc.argtypes = [vp, i64, i64, i64, vp, vp, i64, ctypes.POINTER(i64), vp]
     lib.duo_device_status.argtypes = [vp]
     lib.duo_strerror.argtypes = [i32]
     lib.duo_strerror.restype = ctypes.c_char_p
     for name in ("duo_pack", "duo_sparsify", "duo_spmspv", "duo_spmspv_multi", "duo_free",
-                 "duo_packed_query", "duo_packed_export", "duo_device_status", "duo_abi_version"):
+                 "duo_packed_query", "duo_packed_export", "duo_device_status", "duo_abi_version",
+                 "duo_pack_cmb_noalloc"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -207,3 +209,27 @@ def packed_bytes(h: Packed):
                "duo_packed_export")
         out.append(buf)
     return (info, *out)
+
+
+def duo_pack_cmb_noalloc(W: torch.Tensor, off: torch.Tensor | None = None,
+                         data: torch.Tensor | None = None, stream=None):
+    """Bitmask packing into caller-owned buffers through the entry point that
+    allocates nothing on the device (see duo_pack_cmb_noalloc in
+    include/duo.h).  Missing buffers are allocated here, by the caller side,
+    with PyTorch; returns (off int32 tensor, data uint8 tensor, data bytes)."""
+    if W.dtype != torch.float16 or W.dim() != 2 or not W.is_cuda or W.stride(1) != 1:
+        raise DuoError(DUO_EINVAL, "duo_pack_cmb_noalloc needs a 2-D fp16 CUDA tensor")
+    O, I = W.shape
+    S = (O + 1023) // 1024
+    lib = load_library()
+    if off is None:
+        off = torch.empty(I * S + 1, dtype=torch.int32, device=W.device)
+    nb = ctypes.c_int64(0)
+    st = _stream_ptr(stream)
+    if data is None:
+        _check(lib.duo_pack_cmb_noalloc(W.data_ptr(), O, I, W.stride(0), off.data_ptr(), None, 0,
+                                        ctypes.byref(nb), st), "duo_pack_cmb_noalloc")
+        data = torch.empty(max(16, nb.value), dtype=torch.uint8, device=W.device)
+    _check(lib.duo_pack_cmb_noalloc(W.data_ptr(), O, I, W.stride(0), off.data_ptr(), data.data_ptr(),
+                                    data.numel(), ctypes.byref(nb), st), "duo_pack_cmb_noalloc")
+    return off, data, nb.value
