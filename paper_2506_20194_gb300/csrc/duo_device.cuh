@@ -62,6 +62,23 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Same, but the thread may be suspended for up to hint_ns until the phase
+// completes, so a waiting warp takes no issue slots from the others.
+__device__ __forceinline__ bool mbar_try_wait_suspend(uint64_t* bar, uint32_t parity,
+                                                      uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
+constexpr uint32_t SUSPEND_HINT_NS = 2000;
+
 // Waits for the phase of `parity` with a wall-clock limit.  On timeout the
 // device status word and the CTA's abort flag are set and false returned;
 // a wait also gives up (false) once another warp has raised the abort flag.
@@ -70,7 +87,7 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait_suspend(bar, parity, SUSPEND_HINT_NS)) return true;
     if (*abort_flag) return false;
     if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
       atomicOr(&g_status, STATUS_TIMEOUT);
@@ -134,6 +151,33 @@ __device__ __forceinline__ unsigned int atom_add_acq_rel_gpu(unsigned int* p, un
 
 __device__ __forceinline__ void red_add_release_gpu(unsigned int* p, unsigned int v) {
   asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ int ld_acquire_cta_shared(const int* p) {
+  int v;
+  asm volatile("ld.acquire.cta.shared::cta.b32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release_cta_shared(int* p, int v) {
+  asm volatile("st.release.cta.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
+}
+
+// Spins (bounded, like mbar_wait_bounded) until the shared word at p equals
+// want.  Used to check the exact identity of a ring slot's fill, which an
+// mbarrier parity alone cannot tell apart from a fill two phases earlier.
+__device__ __forceinline__ bool wait_shared_eq(const int* p, int want, volatile int* abort_flag) {
+  if (ld_acquire_cta_shared(p) == want) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    if (ld_acquire_cta_shared(p) == want) return true;
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
+      atomicOr(&g_status, STATUS_TIMEOUT);
+      *abort_flag = 1;
+      return false;
+    }
+  }
 }
 
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
@@ -219,21 +263,23 @@ __device__ inline void load_x_to_smem(uint16_t* xs, const uint16_t* x, int I) {
 }
 
 constexpr int SEL_BINS = 2048;   // histogram of key >> 4
+constexpr int SEL_MAX_WARPS = 32;
 
 // Shared state of the selection.
 struct SelShared {
   uint32_t hist[SEL_BINS];
-  uint32_t sub[16];      // key & 15 inside the threshold bin
-  uint32_t wtot[32];     // per-warp partial sums
-  uint32_t C;            // threshold bin
-  uint32_t aboveC;       // channels in bins above it
+  uint32_t subw[SEL_MAX_WARPS][16];   // per warp: its keys of bin C by key & 15
+  uint32_t wgt[SEL_MAX_WARPS];        // per warp: its keys in bins above C
+  uint32_t wpre[SEL_MAX_WARPS];       // per warp: keys above T | ties << 16 in lower warps
+  uint32_t wown[SEL_MAX_WARPS];       // per warp: its own keys above T | ties << 16
+  uint32_t C, aboveC, T, q;
 };
 
 // Clears the histograms (before the __syncthreads that precedes select_topk).
 __device__ __forceinline__ void select_clear(SelShared* sh) {
   uint4* h = reinterpret_cast<uint4*>(sh->hist);
-  for (int i = threadIdx.x; i < SEL_BINS / 4; i += blockDim.x) h[i] = make_uint4(0u, 0u, 0u, 0u);
-  if (threadIdx.x < 16) sh->sub[threadIdx.x] = 0u;
+  for (int i = threadIdx.x; i < (SEL_BINS + 16 * SEL_MAX_WARPS) / 4; i += blockDim.x)
+    h[i] = make_uint4(0u, 0u, 0u, 0u);   // hist and subw are contiguous
 }
 
 // Exact top-k by magnitude (§3): keeps the k channels with the largest
@@ -243,196 +289,234 @@ __device__ __forceinline__ void select_clear(SelShared* sh) {
 // shared memory (room for a whole number of 32-channel words).
 //
 //  1. histogram of key >> 4 (2048 bins, shared-memory atomics);
-//  2. suffix scan of the histogram (512 threads x 4 bins) to find the bin C
-//     where the count from the top reaches k;
-//  3. histogram of key & 15 over the few channels in bin C, giving the
-//     threshold key T and the count above it; the q = k - count(key > T)
-//     lowest-indexed channels with key == T are kept;
-//  4. every thread builds the "above T" / "equal to T" masks of its own
-//     32-channel words from 16-byte loads of x, a block exclusive scan of the
-//     packed counts orders the words, and the thread writes kb[w] (kept
-//     bitmap, bit b <-> channel 32w+b) and kp[w] (kept channels before word
-//     w; kp[nw] = k);
-//  5. if klist / kvals are given, warps emit klist[r] (channel of kept rank
-//     r, ascending) and kvals[r] (its fp16 bits), lane = bit.
-// Shared-memory accesses are arranged to be bank-conflict free.
+//  2. one warp finds, by suffix scans over 32 blocks of 64 bins and then
+//     over the bins of the block that holds the crossing, the bin C where the
+//     count from the top reaches k;
+//  3. warp w walks its contiguous run of 32-channel words (lane = channel)
+//     and counts its keys in bins above C (ballots) and, by key & 15, its
+//     keys in bin C (its own 16 counters);
+//  4. one warp sums the per-warp counters of bin C to find the threshold
+//     key T = 16 C + b and q = k - count(key > T), the number of channels
+//     with key == T that are kept (the lowest-indexed ones), and scans the
+//     per-warp counts to give every warp the "above T" and "tie" counts
+//     before its own run;
+//  5. warps whose kept ranks meet the requested window walk their words
+//     again: kept channel j has rank r = (channels above T before j) +
+//     min(q, ties before j); if d = (r - r0) mod k is below rn it writes
+//     klist[d] = j and kvals[d] = its fp16 bits.
+//
+// The window is the cyclic rank range r0, r0 + 1, ... (mod k) of length
+// min(rn, k); with r0 = 0 and rn = k the lists are indexed by rank.
 //
 // select_clear() and the loading of xs come first, then a __syncthreads.
-// All threads of the block take part (blockDim.x >= 512, a multiple of 32);
-// it ends with a __syncthreads.
+// All threads of the block take part (512 <= blockDim.x <= 1024, a multiple
+// of 32); it ends with a __syncthreads.
+constexpr uint32_t KEY_NONE = 0xFFFFu;
 __device__ __forceinline__ uint32_t key_of(const uint16_t* xs, int j) { return xs[j] & 0x7FFFu; }
 
-// Masks of the channels of word w (32 channels) above T and equal to T.  The
-// four 16-byte chunks are read in an order rotated by (w >> 1) so that the
-// eight threads of a quarter warp (consecutive words) hit distinct banks.
-__device__ __forceinline__ void word_masks(const uint16_t* xs, int I, int w, bool all, bool none,
-                                           uint32_t T, uint32_t& gt, uint32_t& eq) {
-  const uint4* p = reinterpret_cast<const uint4*>(xs + 32 * w);
-  const int rot = (w >> 1) & 3;
-  gt = 0u;
-  eq = 0u;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int ci = (i + rot) & 3;
-    const uint4 c = p[ci];
-    const uint32_t v[4] = {c.x, c.y, c.z, c.w};
-#pragma unroll
-    for (int h = 0; h < 8; ++h) {
-      const uint32_t key = (v[h >> 1] >> (16 * (h & 1))) & 0x7FFFu;
-      const int b = 8 * ci + h;
-      gt |= (uint32_t)(key > T) << b;
-      eq |= (uint32_t)(key == T) << b;
-    }
-  }
-  const int valid = min(32, I - 32 * w);
-  const uint32_t vmask = valid >= 32 ? FULL_MASK : ((1u << valid) - 1u);
-  if (all) { gt = FULL_MASK; eq = 0u; }
-  if (none) { gt = 0u; eq = 0u; }
-  gt &= vmask;
-  eq &= vmask;
+__device__ __forceinline__ bool ranges_meet(uint32_t a0, uint32_t a1, uint32_t b0, uint32_t b1) {
+  return a0 < b1 && b0 < a1;
 }
 
-__device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t* kb, uint32_t* kp,
+__device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t r0, uint32_t rn,
                                    uint16_t* klist, uint16_t* kvals, SelShared* sh) {
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, wid = tid >> 5;
   const int nwarps = nt >> 5;
   const int nw = (I + 31) >> 5;
-  const bool all = k >= I, none = k <= 0;
-  uint32_t T = 0u;
-  int q = 0;
-  if (!all && !none) {
-    // 1. histogram of the high 11 key bits
-    {
-      int j = tid;
-      for (; j + 3 * nt < I; j += 4 * nt) {
-        const uint32_t k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
-        const uint32_t k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
-        atomicAdd(&sh->hist[k0 >> 4], 1u);
-        atomicAdd(&sh->hist[k1 >> 4], 1u);
-        atomicAdd(&sh->hist[k2 >> 4], 1u);
-        atomicAdd(&sh->hist[k3 >> 4], 1u);
-      }
-      for (; j < I; j += nt) atomicAdd(&sh->hist[key_of(xs, j) >> 4], 1u);
-    }
+  const uint32_t kk = (uint32_t)k;
+  const bool whole = rn >= kk;
+  // list position of rank r, or -1 outside the window
+  auto slot_of = [&](uint32_t r) -> int {
+    const uint32_t d = r >= r0 ? r - r0 : r + kk - r0;
+    return (whole || d < rn) ? (int)d : -1;
+  };
+  if (k <= 0) {   // nothing kept
     __syncthreads();
-    // 2. suffix scan: thread t < 512 owns bins [4t, 4t + 4)
-    uint32_t c[4] = {0u, 0u, 0u, 0u}, s = 0, incl = 0;
-    if (tid < 512) {
-      const uint4 h = reinterpret_cast<const uint4*>(sh->hist)[tid];
-      c[0] = h.x; c[1] = h.y; c[2] = h.z; c[3] = h.w;
-      s = c[0] + c[1] + c[2] + c[3];
-      incl = s;   // suffix over lanes >= lane inside the warp
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t t = __shfl_down_sync(FULL_MASK, incl, o);
-        if (lane + o < 32) incl += t;
-      }
-      if (lane == 0) sh->wtot[wid] = incl;
-    }
-    __syncthreads();
-    if (tid < 512) {
-      uint32_t above_w = (lane > wid && lane < 16) ? sh->wtot[lane] : 0u;
-      above_w = __reduce_add_sync(FULL_MASK, above_w);
-      const uint32_t hi = above_w + incl;   // channels in bins >= 4*tid
-      const uint32_t lo = hi - s;           // channels in bins >= 4*tid + 4
-      if (lo < (uint32_t)k && (uint32_t)k <= hi) {
-        uint32_t acc = lo;
-        int b = 0;
-#pragma unroll
-        for (int i = 3; i >= 0; --i) {
-          if (acc + c[i] >= (uint32_t)k) { b = i; break; }
-          acc += c[i];
-        }
-        sh->C = 4u * tid + (uint32_t)b;
-        sh->aboveC = acc;
-      }
-    }
-    __syncthreads();
-    // 3. the 16 keys of bin C (few channels: contention-free atomics)
-    const uint32_t C = sh->C;
+    return;
+  }
+  if (k >= I) {   // everything kept: rank = channel
     for (int j = tid; j < I; j += nt) {
-      const uint32_t key = key_of(xs, j);
-      if ((key >> 4) == C) atomicAdd(&sh->sub[key & 15u], 1u);
-    }
-    __syncthreads();
-    uint32_t sub[16];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint4 v = reinterpret_cast<const uint4*>(sh->sub)[i];
-      sub[4 * i] = v.x; sub[4 * i + 1] = v.y; sub[4 * i + 2] = v.z; sub[4 * i + 3] = v.w;
-    }
-    uint32_t above = sh->aboveC;
-    int b = -1;
-#pragma unroll
-    for (int v = 15; v >= 0; --v) {
-      if (b < 0) {
-        if (above + sub[v] >= (uint32_t)k) b = v;
-        else above += sub[v];
+      const int d = slot_of((uint32_t)j);
+      if (d >= 0) {
+        if (klist != nullptr) klist[d] = (uint16_t)j;
+        if (kvals != nullptr) kvals[d] = xs[j];
       }
     }
-    if (b < 0) b = 0;
-    T = 16u * C + (uint32_t)b;
-    q = k - (int)above;
+    __syncthreads();
+    return;
   }
-  // 4. thread tid owns words [w0, w1)
-  const int per = (nw + nt - 1) / nt;
-  const int w0 = min(nw, tid * per), w1 = min(nw, w0 + per);
-  uint32_t packed = 0;   // greater-count | tie-count << 16 (each <= 65535)
-  for (int w = w0; w < w1; ++w) {
-    uint32_t gt, eq;
-    word_masks(xs, I, w, all, none, T, gt, eq);
-    kb[w] = gt;   // provisional: the masks are kept in kb / kp until ranked
-    kp[w] = eq;
-    packed += (uint32_t)__popc(gt) | ((uint32_t)__popc(eq) << 16);
+  // 1. histogram of the high 11 key bits (4 independent loads in flight)
+  {
+    int j = tid;
+    for (; j + 3 * nt < I; j += 4 * nt) {
+      const uint32_t k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
+      const uint32_t k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
+      atomicAdd(&sh->hist[k0 >> 4], 1u);
+      atomicAdd(&sh->hist[k1 >> 4], 1u);
+      atomicAdd(&sh->hist[k2 >> 4], 1u);
+      atomicAdd(&sh->hist[k3 >> 4], 1u);
+    }
+    for (; j < I; j += nt) atomicAdd(&sh->hist[key_of(xs, j) >> 4], 1u);
   }
-  const uint32_t inc = warp_inclusive_scan(packed, lane);
-  if (lane == 31) sh->wtot[wid] = inc;   // step 2's wtot reads ended two barriers ago
   __syncthreads();
+  // 2. threshold bin C, by warp 0 alone: lane l totals bins [64 l, 64 l + 64),
+  //    a suffix scan over lanes finds the lane whose bins hold the crossing,
+  //    and a second scan over that lane's 64 bins (2 per lane) finds C.
   if (wid == 0) {
-    uint32_t t = lane < nwarps ? sh->wtot[lane] : 0u;
-    t = warp_inclusive_scan(t, lane);
-    sh->wtot[lane] = t;
+    const uint4* h4 = reinterpret_cast<const uint4*>(sh->hist) + 16 * lane;
+    uint32_t s64 = 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const uint4 h = h4[(i + lane) & 15];   // rotated: a quarter warp hits 8 bank groups
+      s64 += (h.x + h.y) + (h.z + h.w);
+    }
+    uint32_t sl = s64;   // keys in bins >= 64 * lane
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t t = __shfl_down_sync(FULL_MASK, sl, o);
+      if (lane + o < 32) sl += t;
+    }
+    const int L = 31 - __clz(__ballot_sync(FULL_MASK, sl >= kk));
+    const uint32_t above_l = __shfl_sync(FULL_MASK, sl - s64, L);   // keys in bins >= 64 (L + 1)
+    const uint2 h2 = reinterpret_cast<const uint2*>(sh->hist)[32 * L + lane];   // bins 64 L + 2 lane, +1
+    const uint32_t s2 = h2.x + h2.y;
+    uint32_t sp = s2;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t t = __shfl_down_sync(FULL_MASK, sp, o);
+      if (lane + o < 32) sp += t;
+    }
+    const int M = 31 - __clz(__ballot_sync(FULL_MASK, above_l + sp >= kk));
+    if (lane == M) {
+      const uint32_t above = above_l + sp - s2;   // keys above bin 64 L + 2 M + 1
+      const bool hi = above + h2.y >= kk;
+      sh->C = 64u * (uint32_t)L + 2u * (uint32_t)M + (hi ? 1u : 0u);
+      sh->aboveC = hi ? above : above + h2.y;
+    }
   }
   __syncthreads();
-  const uint32_t base = (wid > 0 ? sh->wtot[wid - 1] : 0u) + inc - packed;
-  uint32_t gpre = base & 0xFFFFu, epre = base >> 16;
-  for (int w = w0; w < w1; ++w) {
-    const uint32_t gt = kb[w], eq = kp[w];
-    const int allowed = q - (int)epre;
-    uint32_t take = 0u;
-    if (allowed > 0 && eq != 0u)
-      take = allowed >= __popc(eq) ? eq : (eq & ((1u << select_bit(eq, allowed)) - 1u));
-    kb[w] = gt | take;
-    kp[w] = gpre + min(epre, (uint32_t)q);
-    gpre += __popc(gt);
-    epre += __popc(eq);
-  }
-  if (tid == 0) kp[nw] = all ? (uint32_t)I : (none ? 0u : (uint32_t)k);
-  __syncthreads();
-  // 5. warp-parallel emission of the kept list
-  if (klist != nullptr || kvals != nullptr) {
-    const uint32_t lt = (1u << lane) - 1u;
-    for (int w = wid; w < nw; w += nwarps) {
-      const uint32_t kbw = kb[w];
-      if ((kbw >> lane) & 1u) {
-        const uint32_t rank = kp[w] + __popc(kbw & lt);
-        const int j = 32 * w + lane;
-        if (klist != nullptr) klist[rank] = (uint16_t)j;
-        if (kvals != nullptr) kvals[rank] = xs[j];
+  // 3. per-warp counts over the warp's words [w0, w1)
+  const int per = (nw + nwarps - 1) / nwarps;
+  const int w0 = min(nw, wid * per), w1 = min(nw, w0 + per);
+  {
+    const uint32_t C = sh->C;
+    uint32_t ngt = 0;
+    for (int w = w0; w < w1; w += 4) {
+      uint32_t key[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int j = 32 * (w + u) + lane;
+        key[u] = (w + u < w1 && j < I) ? key_of(xs, j) : KEY_NONE;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const bool valid = key[u] != KEY_NONE;
+        ngt += (uint32_t)__popc(__ballot_sync(FULL_MASK, valid && (key[u] >> 4) > C));
+        if (valid && (key[u] >> 4) == C) atomicAdd(&sh->subw[wid][key[u] & 15u], 1u);
       }
     }
-    __syncthreads();
+    if (lane == 0) sh->wgt[wid] = ngt;
   }
-}
-
-// Channel id of kept index i (0 <= i < kp[nw]) from the bitmap + prefix.
-__device__ __forceinline__ int kept_channel(const uint32_t* kb, const uint32_t* kp, int nw, uint32_t i) {
-  int lo = 0, hi = nw - 1;   // find the last w with kp[w] <= i
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (kp[mid] <= i) lo = mid; else hi = mid - 1;
+  __syncthreads();
+  // 4. by warp 0 alone: the threshold key T = 16 C + b (lane v < 16 = key & 15
+  //    inside bin C), q, and for every warp w (lane w) its own and its lower
+  //    warps' counts above T and equal to T.
+  if (wid == 0) {
+    uint32_t part[4] = {0u, 0u, 0u, 0u};
+    if (lane < 16) {
+#pragma unroll
+      for (int w = 0; w < SEL_MAX_WARPS; ++w)
+        if (w < nwarps) part[w & 3] += sh->subw[w][lane];
+    }
+    const uint32_t sv = (part[0] + part[1]) + (part[2] + part[3]);
+    uint32_t suf = sv;   // keys of bin C with key & 15 >= lane
+#pragma unroll
+    for (int o = 1; o < 16; o <<= 1) {
+      const uint32_t t = __shfl_down_sync(FULL_MASK, suf, o);
+      if (lane + o < 16) suf += t;
+    }
+    const uint32_t need = kk - sh->aboveC;   // >= 1, <= hist[C]
+    const int b = 31 - __clz(__ballot_sync(FULL_MASK, lane < 16 && suf >= need));
+    const uint32_t above_in_c = __shfl_sync(FULL_MASK, suf - sv, b);
+    uint32_t al = 0, tl = 0;
+    if (lane < nwarps) {
+      const uint4* row = reinterpret_cast<const uint4*>(sh->subw[lane]);
+      al = sh->wgt[lane];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int c = (i + (lane >> 1)) & 3;   // rotated: conflict-free quarter warps
+        const uint4 r4 = row[c];
+        const uint32_t v4[4] = {r4.x, r4.y, r4.z, r4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int v = 4 * c + e;
+          al += v > b ? v4[e] : 0u;
+          tl += v == b ? v4[e] : 0u;
+        }
+      }
+    }
+    const uint32_t own = al | (tl << 16);   // each <= 65535
+    const uint32_t pre = warp_inclusive_scan(own, lane) - own;
+    if (lane < nwarps) {
+      sh->wpre[lane] = pre;
+      sh->wown[lane] = own;
+    }
+    if (lane == 0) {
+      sh->T = 16u * sh->C + (uint32_t)b;
+      sh->q = need - above_in_c;   // >= 1
+    }
   }
-  return 32 * lo + select_bit(kb[lo], (int)(i - kp[lo]));
+  __syncthreads();
+  const uint32_t T = sh->T, q = sh->q;
+  uint32_t gpre, epre, a_own, t_own;
+  {
+    const uint32_t pre = sh->wpre[wid], own = sh->wown[wid];
+    gpre = pre & 0xFFFFu;
+    epre = pre >> 16;
+    a_own = own & 0xFFFFu;
+    t_own = own >> 16;
+  }
+  // 5. emission by the warps whose kept ranks meet the window
+  if (klist != nullptr || kvals != nullptr) {
+    const uint32_t R = gpre + min(epre, q);
+    const uint32_t Kw = a_own + min(epre + t_own, q) - min(epre, q);
+    bool meet = whole;
+    if (!meet && Kw > 0) {
+      const uint32_t e0 = r0 + rn;   // window [r0, e0), wrapping past kk
+      meet = ranges_meet(R, R + Kw, r0, min(e0, kk)) || (e0 > kk && ranges_meet(R, R + Kw, 0u, e0 - kk));
+    }
+    if (meet) {
+      const uint32_t lt = (1u << lane) - 1u;
+      for (int w = w0; w < w1; w += 4) {
+        uint32_t key[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int j = 32 * (w + u) + lane;
+          key[u] = (w + u < w1 && j < I) ? key_of(xs, j) : KEY_NONE;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const bool valid = key[u] != KEY_NONE;
+          const bool isg = valid && key[u] > T;
+          const bool ise = valid && key[u] == T;
+          const uint32_t g = __ballot_sync(FULL_MASK, isg);
+          const uint32_t e = __ballot_sync(FULL_MASK, ise);
+          const uint32_t tr = epre + (uint32_t)__popc(e & lt);   // ties before this channel
+          if (isg || (ise && tr < q)) {
+            const int d = slot_of(gpre + (uint32_t)__popc(g & lt) + min(tr, q));
+            if (d >= 0) {
+              const int j = 32 * (w + u) + lane;
+              if (klist != nullptr) klist[d] = (uint16_t)j;
+              if (kvals != nullptr) kvals[d] = xs[j];
+            }
+          }
+          gpre += (uint32_t)__popc(g);
+          epre += (uint32_t)__popc(e);
+        }
+      }
+    }
+  }
+  __syncthreads();
 }
 
 }  // namespace duo

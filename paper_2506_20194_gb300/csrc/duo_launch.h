@@ -32,7 +32,9 @@ struct CmbArgs {
                          // between launches; owned by the first handle
   int slot_bytes;        // in: largest record of the launch's weights (bytes);
                          // the launcher rounds it and picks the slot count
-  int nslot;             // set by the launcher
+  int nslot;             // set by the launcher (a multiple of the consumer count)
+  int group;             // set by the launcher: records a consumer waits for at once
+  int list_cap;          // set by the launcher: kept-list entries a CTA emits
 };
 
 struct Idx16Args {

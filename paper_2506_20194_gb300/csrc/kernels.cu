@@ -293,17 +293,15 @@ cudaError_t launch_idx16_offsets(const uint32_t* cnt_js, int64_t I, int S, uint3
 constexpr int SPARSIFY_THREADS = 1024;
 
 struct SelLayout {
-  size_t xs, kb, kp, klist, sel, end;
+  size_t xs, klist, sel, end;
 };
 
-__host__ __device__ inline SelLayout sel_layout(int I, size_t base, bool with_list) {
-  const size_t nw = (size_t)(I + 31) / 32;
+// list_entries: room for that many kept-list entries in shared memory (0: none).
+__host__ __device__ inline SelLayout sel_layout(int I, size_t base, int list_entries) {
   SelLayout L;
   size_t o = base;
   L.xs = o;    o += align_up(2 * (size_t)I, 64);   // whole 32-channel words
-  L.kb = o;    o += align_up(4 * nw, 16);
-  L.kp = o;    o += align_up(4 * (nw + 1), 16);
-  L.klist = o; if (with_list) o += align_up(2 * (size_t)I, 16);
+  L.klist = o; o += align_up(2 * (size_t)list_entries, 16);
   L.sel = o;   o += align_up(sizeof(SelShared), 16);
   L.end = o;
   return L;
@@ -314,19 +312,18 @@ __global__ void __launch_bounds__(SPARSIFY_THREADS) sparsify_kernel(const uint16
                                                                     uint16_t* __restrict__ kidx,
                                                                     uint16_t* __restrict__ kval) {
   extern __shared__ __align__(128) uint8_t sm[];
-  const SelLayout L = sel_layout(I, 0, false);
+  const SelLayout L = sel_layout(I, 0, 0);
   uint16_t* xs = reinterpret_cast<uint16_t*>(sm + L.xs);
   SelShared* sel = reinterpret_cast<SelShared*>(sm + L.sel);
   load_x_to_smem(xs, x, I);
   select_clear(sel);
   __syncthreads();
-  select_topk(xs, I, k, reinterpret_cast<uint32_t*>(sm + L.kb),
-              reinterpret_cast<uint32_t*>(sm + L.kp), kidx, kval, sel);
+  select_topk(xs, I, k, 0u, (uint32_t)k, kidx, kval, sel);
 }
 
 cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uint16_t* kval,
                             cudaStream_t st) {
-  const size_t smem = sel_layout(I, 0, false).end;
+  const size_t smem = sel_layout(I, 0, 0).end;
   cudaError_t e = cudaFuncSetAttribute(sparsify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
@@ -346,7 +343,11 @@ cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uin
 // record offset and size; the next PQ-1 items of the lane are resolved ahead
 // so their offset loads are in flight) and issues a 1-D bulk copy of each
 // record into ring slot v % nslot, signalled on the slot's "full" mbarrier
-// with the byte count.  Slots are as large as the largest record of the
+// with the byte count.  Every slot carries the index of the item it holds
+// (tag, written by the producer) and of the item last consumed from it (rel,
+// written by the consumer); each side checks the exact index before relying
+// on the mbarrier, whose parity cannot tell a fill from one two phases
+// earlier.  Slots are as large as the largest record of the
 // launch's weights (about 1.3 KB at 50% weight density), so the ring holds
 // as many records as the shared memory allows.
 //
@@ -364,26 +365,27 @@ cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uin
 // before its first reduction into y.  The launch is cooperative, so all CTAs
 // are co-resident and the barrier cannot deadlock.
 // ------------------------------------------------------------------------
-constexpr int CMB_NC = 16;
+constexpr int CMB_NC = 15;   // 16 warps in all: 4 per scheduler, up to 128 registers
 constexpr int CMB_THREADS = 32 * (1 + CMB_NC);
 constexpr int CMB_MAX_SLOTS = 256;
 
 struct CmbLayout {
   SelLayout sel;
-  size_t tile, full, empty, meta, ring, total;
+  size_t tile, full, empty, xval, ring, total;
 };
 
-__host__ __device__ inline CmbLayout cmb_layout(int I, bool fused, int nslot, int slot_bytes) {
+__host__ __device__ inline CmbLayout cmb_layout(int I, bool fused, int list_cap, int nslot,
+                                                int slot_bytes) {
   CmbLayout L;
   size_t o = 0;
   if (fused) {
-    L.sel = sel_layout(I, 0, true);
+    L.sel = sel_layout(I, 0, list_cap);
     o = L.sel.end;
   }
   L.tile = o;  o += 2 * SEG_ROWS * sizeof(float);
   L.full = o;  o += 8 * (size_t)nslot;
   L.empty = o; o += 8 * (size_t)nslot;
-  L.meta = o;  o += align_up(4 * (size_t)nslot, 16);
+  L.xval = o;  o += align_up(4 * (size_t)nslot, 16);
   o = align_up(o, 128);
   L.ring = o;  o += (size_t)nslot * slot_bytes;
   L.total = o;
@@ -412,6 +414,34 @@ __device__ __forceinline__ void decode_two(const uint8_t* ra, uint16_t xa, const
     if (mb & (1u << t)) {
       acc[t] = fma_f16_f32(*pb, xb, acc[t]);
       ++pb;
+    }
+  }
+}
+
+// Four records of the same segment at once (two packed prefix sums, four
+// independent load chains per bit position).
+__device__ __forceinline__ void decode_four(const uint8_t* const (&r)[4], const uint16_t (&xv)[4],
+                                            float (&acc)[32], int lane) {
+  uint32_t m[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) m[i] = reinterpret_cast<const uint32_t*>(r[i])[lane];
+  const uint32_t c01 = (uint32_t)__popc(m[0]) | ((uint32_t)__popc(m[1]) << 16);
+  const uint32_t c23 = (uint32_t)__popc(m[2]) | ((uint32_t)__popc(m[3]) << 16);
+  const uint32_t e01 = warp_inclusive_scan(c01, lane) - c01;
+  const uint32_t e23 = warp_inclusive_scan(c23, lane) - c23;
+  const uint16_t* p[4] = {
+      reinterpret_cast<const uint16_t*>(r[0] + MASK_BYTES) + (e01 & 0xFFFFu),
+      reinterpret_cast<const uint16_t*>(r[1] + MASK_BYTES) + (e01 >> 16),
+      reinterpret_cast<const uint16_t*>(r[2] + MASK_BYTES) + (e23 & 0xFFFFu),
+      reinterpret_cast<const uint16_t*>(r[3] + MASK_BYTES) + (e23 >> 16)};
+#pragma unroll
+  for (int t = 0; t < 32; ++t) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (m[i] & (1u << t)) {
+        acc[t] = fma_f16_f32(*p[i], xv[i], acc[t]);
+        ++p[i];
+      }
     }
   }
 }
@@ -469,33 +499,41 @@ struct SlotCursor {
   }
 };
 
+// Where an item's record lives.  The two offset loads stay in flight until
+// the item is issued, PQ rounds later: nothing here reads their results, so
+// the producer never waits a memory latency per round.
 struct Resolved {
-  const uint8_t* src;
-  uint32_t bytes;
+  const uint8_t* data;   // the product's packed data
+  uint32_t o0, o1;       // off[j * S + s], off[j * S + s + 1] (16-byte units)
   uint16_t xb;
-  bool bad;
+  bool bad_j;            // channel id out of range
+  __device__ __forceinline__ uint32_t bytes() const { return (o1 - o0) * 16u; }
+  __device__ __forceinline__ bool bad(int slot_bytes) const {
+    const uint32_t b = bytes();
+    return bad_j || o1 < o0 || b < (uint32_t)MASK_BYTES || b > (uint32_t)slot_bytes;
+  }
 };
 
 template <bool FUSED>
 __device__ __forceinline__ Resolved resolve_item(const CmbArgs& a, const ItemCursor& c,
-                                                 const uint16_t* klist, const uint16_t* xs) {
+                                                 const uint16_t* klist, const uint16_t* xs, int r0) {
   Resolved r;
   int j;
   if (FUSED) {
-    j = klist[c.i];
+    const int d = c.i >= r0 ? c.i - r0 : c.i + a.k - r0;   // position in this CTA's list window
+    j = klist[d];
     r.xb = xs[j];
   } else {
     j = __ldg(a.kidx + c.i);
     r.xb = __ldg(a.kval + c.i);
   }
-  r.bad = j >= a.I;
-  if (r.bad) j = 0;   // keep the loads below in bounds; the item is rejected
+  r.bad_j = j >= a.I;
+  if (r.bad_j) j = 0;   // keep the loads below in bounds; the item is rejected
   const CmbProb& P = a.p[c.p];
   const int64_t ri = (int64_t)j * P.S + c.s;
-  const uint32_t o0 = __ldg(P.off + ri), o1 = __ldg(P.off + ri + 1);
-  r.bytes = (o1 - o0) * 16u;
-  r.src = P.data + (size_t)o0 * 16;
-  r.bad = r.bad || o1 < o0 || r.bytes < (uint32_t)MASK_BYTES || r.bytes > (uint32_t)a.slot_bytes;
+  r.o0 = __ldg(P.off + ri);
+  r.o1 = __ldg(P.off + ri + 1);
+  r.data = P.data;
   return r;
 }
 
@@ -505,15 +543,13 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   __shared__ volatile int abort_flag;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nslot = a.nslot, slot_bytes = a.slot_bytes;
-  const CmbLayout L = cmb_layout(a.I, FUSED, nslot, slot_bytes);
+  const CmbLayout L = cmb_layout(a.I, FUSED, a.list_cap, nslot, slot_bytes);
   float* tile = reinterpret_cast<float*>(sm + L.tile);
   uint64_t* full = reinterpret_cast<uint64_t*>(sm + L.full);
   uint64_t* empty = reinterpret_cast<uint64_t*>(sm + L.empty);
-  uint32_t* meta = reinterpret_cast<uint32_t*>(sm + L.meta);
+  uint32_t* xval = reinterpret_cast<uint32_t*>(sm + L.xval);
   uint8_t* ring = sm + L.ring;
   uint16_t* xs = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.xs) : nullptr;
-  uint32_t* kb = FUSED ? reinterpret_cast<uint32_t*>(sm + L.sel.kb) : nullptr;
-  uint32_t* kp = FUSED ? reinterpret_cast<uint32_t*>(sm + L.sel.kp) : nullptr;
   uint16_t* klist = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.klist) : nullptr;
   SelShared* sel = FUSED ? reinterpret_cast<SelShared*>(sm + L.sel.sel) : nullptr;
 
@@ -548,18 +584,25 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       base += a.p[p].O;
     }
   }
-  __syncthreads();
-  if (FUSED) select_topk(xs, a.I, a.k, kb, kp, klist, nullptr, sel);
-
   int64_t total = 0;
   for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
   const int64_t u0 = total * blockIdx.x / gridDim.x;
   const int64_t u1 = total * (blockIdx.x + 1) / gridDim.x;
   const int nv = (int)(u1 - u0);
+  // This CTA's items use the kept ranks r0, r0 + 1, ... (mod k): only those
+  // entries of the kept list are emitted, at positions 0, 1, ...
+  int r0 = 0;
+  if (FUSED) {
+    ItemCursor first;
+    first.set(a, u0);
+    r0 = first.i;
+  }
+  __syncthreads();
+  if (FUSED) select_topk(xs, a.I, a.k, (uint32_t)r0, (uint32_t)a.list_cap, klist, nullptr, sel);
 
   if (warp == 0) {
     // ---------------- producer ----------------
-    constexpr int PQ = 4;
+    constexpr int PQ = 8;
     const uint64_t pol = policy_evict_first();
     int last_v = -1;
     bool stop = false;
@@ -572,17 +615,22 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     for (int d = 0; d < PQ; ++d) {
       if (lane + 32 * d < nv) {
         if (d > 0) cur.advance(a, 32);
-        q[d] = resolve_item<FUSED>(a, cur, klist, xs);
+        q[d] = resolve_item<FUSED>(a, cur, klist, xs, r0);
       }
     }
-    for (int v0 = lane; v0 < nv && !stop; v0 += 32 * PQ) {
+    // Rounds of 32 items: round R issues items 32 R .. 32 R + 31, lane l the
+    // item 32 R + l.  A __syncwarp opens every round, so the rounds run in
+    // lockstep and items are issued in increasing round order.
+    for (int R0 = 0; R0 < nv; R0 += 32 * PQ) {
 #pragma unroll
       for (int d = 0; d < PQ; ++d) {
-        const int v = v0 + 32 * d;
-        if (stop || v >= nv) continue;
-        if (abort_flag) { stop = true; continue; }
+        __syncwarp();
+        stop = __any_sync(FULL_MASK, stop || abort_flag != 0);
+        if (stop) break;
+        const int v = R0 + 32 * d + lane;
+        if (v >= nv) continue;
         const Resolved r = q[d];
-        if (r.bad) {
+        if (r.bad(slot_bytes)) {
           atomicOr(&g_status, STATUS_FORMAT);
           abort_flag = 1;
           stop = true;
@@ -590,18 +638,23 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
         }
         if (v + 32 * PQ < nv) {                 // refill: this lane's item v + 32*PQ
           cur.advance(a, 32);
-          q[d] = resolve_item<FUSED>(a, cur, klist, xs);
+          q[d] = resolve_item<FUSED>(a, cur, klist, xs, r0);
         }
+        // Fill n of a slot waits until fill n - 1 has been consumed.  Fill
+        // n - 1 was issued in an earlier round (nslot >= 32), after fill
+        // n - 2 had been released, so the "empty" phase parity is exact.
         if (sc.n > 0 && !mbar_wait_bounded(&empty[sc.slot], (uint32_t)((sc.n - 1) & 1), &abort_flag)) {
           stop = true;
           continue;
         }
-        meta[sc.slot] = r.xb;
-        mbar_arrive_expect_tx(&full[sc.slot], r.bytes);
-        bulk_g2s(ring + (size_t)sc.slot * slot_bytes, r.src, r.bytes, &full[sc.slot], pol);
+        xval[sc.slot] = r.xb;
+        mbar_arrive_expect_tx(&full[sc.slot], r.bytes());
+        bulk_g2s(ring + (size_t)sc.slot * slot_bytes, r.data + (size_t)r.o0 * 16, r.bytes(),
+                 &full[sc.slot], pol);
         last_v = v;
         sc.advance(32, nslot);
       }
+      if (stop) break;
     }
     if (abort_flag) {
       // Let this lane's copies still in flight land before the CTA exits.
@@ -627,6 +680,15 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       }
     }
     float acc[32];
+    // Item v sits in slot v % nslot.  nslot is a multiple of CMB_NC, so a
+    // slot only ever holds items of this consumer, which it takes in
+    // increasing order and releases before waiting on any item nslot later
+    // (group * CMB_NC <= nslot): when it waits for fill n, fill n - 1 is
+    // consumed and fill n + 1 not yet issued, so the "full" parity is exact.
+    auto wait_item = [&](const SlotCursor& q) -> bool {
+      return mbar_wait_bounded(&full[q.slot], (uint32_t)(q.n & 1), &abort_flag);
+    };
+    auto release = [&](const SlotCursor& q) { mbar_arrive(&empty[q.slot]); };
     int64_t u = u0;
     int piece = 0;
     while (u < u1) {
@@ -639,31 +701,60 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       for (int t = 0; t < 32; ++t) acc[t] = 0.f;
       bool any = false;
       int v = va + ((c - va % CMB_NC) % CMB_NC + CMB_NC) % CMB_NC;
+      // this consumer's items four at a time, then in pairs, then alone
+      if (a.group >= 4) {
+        for (; v + 3 * CMB_NC < vb; v += 4 * CMB_NC) {
+          SlotCursor q4[4];
+          bool ok = !abort_flag;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            q4[i].set(v + i * CMB_NC, nslot);
+            ok = ok && wait_item(q4[i]);
+          }
+          if (ok) {
+            const uint8_t* const rr[4] = {ring + (size_t)q4[0].slot * slot_bytes,
+                                          ring + (size_t)q4[1].slot * slot_bytes,
+                                          ring + (size_t)q4[2].slot * slot_bytes,
+                                          ring + (size_t)q4[3].slot * slot_bytes};
+            const uint16_t xv[4] = {(uint16_t)xval[q4[0].slot], (uint16_t)xval[q4[1].slot],
+                                    (uint16_t)xval[q4[2].slot], (uint16_t)xval[q4[3].slot]};
+            decode_four(rr, xv, acc, lane);
+            any = true;
+          }
+          __syncwarp();
+          if (lane == 0) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) release(q4[i]);
+          }
+        }
+      }
       SlotCursor sc, sc2;
       sc.set(v, nslot);
-      sc2.set(v + CMB_NC, nslot);
-      for (; v + CMB_NC < vb; v += 2 * CMB_NC) {   // this consumer's items in pairs
-        if (!abort_flag && mbar_wait_bounded(&full[sc.slot], (uint32_t)(sc.n & 1), &abort_flag) &&
-            mbar_wait_bounded(&full[sc2.slot], (uint32_t)(sc2.n & 1), &abort_flag)) {
-          decode_two(ring + (size_t)sc.slot * slot_bytes, (uint16_t)meta[sc.slot],
-                     ring + (size_t)sc2.slot * slot_bytes, (uint16_t)meta[sc2.slot], acc, lane);
-          any = true;
+      if (a.group >= 2) {
+        sc2.set(v + CMB_NC, nslot);
+        for (; v + CMB_NC < vb; v += 2 * CMB_NC) {   // pairs
+          if (!abort_flag && wait_item(sc) && wait_item(sc2)) {
+            decode_two(ring + (size_t)sc.slot * slot_bytes, (uint16_t)xval[sc.slot],
+                       ring + (size_t)sc2.slot * slot_bytes, (uint16_t)xval[sc2.slot], acc, lane);
+            any = true;
+          }
+          __syncwarp();
+          if (lane == 0) {
+            release(sc);
+            release(sc2);
+          }
+          sc.advance(2 * CMB_NC, nslot);
+          sc2.advance(2 * CMB_NC, nslot);
         }
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&empty[sc.slot]);
-          mbar_arrive(&empty[sc2.slot]);
-        }
-        sc.advance(2 * CMB_NC, nslot);
-        sc2.advance(2 * CMB_NC, nslot);
       }
-      if (v < vb) {
-        if (!abort_flag && mbar_wait_bounded(&full[sc.slot], (uint32_t)(sc.n & 1), &abort_flag)) {
-          decode_record(ring + (size_t)sc.slot * slot_bytes, (uint16_t)meta[sc.slot], acc, lane);
+      for (; v < vb; v += CMB_NC) {   // singles
+        if (!abort_flag && wait_item(sc)) {
+          decode_record(ring + (size_t)sc.slot * slot_bytes, (uint16_t)xval[sc.slot], acc, lane);
           any = true;
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[sc.slot]);
+        if (lane == 0) release(sc);
+        sc.advance(CMB_NC, nslot);
       }
       float* tb = tile + (piece & 1) * SEG_ROWS;
       if (any) {
@@ -674,6 +765,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
         // First reduction into y: every CTA must have zeroed its slice.
         const uint64_t t0 = globaltimer_ns();
         while (ld_acquire_gpu(a.bar + 1) == gen0) {
+          __nanosleep(64);
           if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
             atomicOr(&g_status, STATUS_TIMEOUT);
             abort_flag = 1;
@@ -721,19 +813,25 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   if (total <= 0) return cudaSuccess;
   const int grid = (int)std::min<int64_t>(dp.nsm, total);
   if ((total + grid - 1) / grid >= (int64_t)1 << 30) return cudaErrorInvalidValue;
+  // Kept-list window of a CTA: at most its item count, at most k.
+  const int64_t per_cta = (total + grid - 1) / grid;
+  a.list_cap = fused ? (int)std::min<int64_t>(per_cta, a.k) : 0;
   // Slot size: the largest record among the launch's weights (given by the
-  // caller in a.slot_bytes); slot count: as many as the shared memory holds.
+  // caller in a.slot_bytes); slot count: as many as the shared memory holds,
+  // a multiple of the consumer count.
   const int slot_bytes = (int)align_up((size_t)std::max(a.slot_bytes, MASK_BYTES + 16), 16);
   if (slot_bytes > MAX_RECORD_BYTES) return cudaErrorInvalidValue;
   const size_t avail = (size_t)dp.smem_optin - 256;   // static shared memory headroom
-  const size_t fixed = cmb_layout(a.I, fused, 0, slot_bytes).total + 128;
+  const size_t fixed = cmb_layout(a.I, fused, a.list_cap, 0, slot_bytes).total + 128;
   if (fixed >= avail) return cudaErrorInvalidValue;
   int nslot = (int)((avail - fixed) / (slot_bytes + 20));
   nslot = std::min(nslot, CMB_MAX_SLOTS);
-  if (nslot < 32) return cudaErrorInvalidValue;
+  nslot -= nslot % CMB_NC;
+  if (nslot < std::max(32, CMB_NC)) return cudaErrorInvalidValue;
+  a.group = nslot >= 4 * CMB_NC ? 4 : (nslot >= 2 * CMB_NC ? 2 : 1);
   a.nslot = nslot;
   a.slot_bytes = slot_bytes;
-  const size_t smem = cmb_layout(a.I, fused, nslot, slot_bytes).total;
+  const size_t smem = cmb_layout(a.I, fused, a.list_cap, nslot, slot_bytes).total;
   void (*kern)(const CmbArgs) = fused ? cmb_spmspv_kernel<true> : cmb_spmspv_kernel<false>;
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
@@ -762,7 +860,7 @@ template <bool FUSED>
 __global__ void __launch_bounds__(IDX16_THREADS, 1) idx16_spmspv_kernel(const Idx16Args a) {
   extern __shared__ __align__(128) uint8_t sm[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const SelLayout L = sel_layout(a.I, 0, true);
+  const SelLayout L = sel_layout(a.I, 0, a.I);
   uint16_t* xs = reinterpret_cast<uint16_t*>(sm + L.xs);
   uint16_t* klist = reinterpret_cast<uint16_t*>(sm + L.klist);
   if (FUSED) {
@@ -770,8 +868,7 @@ __global__ void __launch_bounds__(IDX16_THREADS, 1) idx16_spmspv_kernel(const Id
     load_x_to_smem(xs, a.x, a.I);
     select_clear(sel);
     __syncthreads();
-    select_topk(xs, a.I, a.k, reinterpret_cast<uint32_t*>(sm + L.kb),
-                reinterpret_cast<uint32_t*>(sm + L.kp), klist, nullptr, sel);
+    select_topk(xs, a.I, a.k, 0u, (uint32_t)a.k, klist, nullptr, sel);
   }
   const int nwt = gridDim.x * (IDX16_THREADS / 32);
   for (int i = blockIdx.x * (IDX16_THREADS / 32) + warp; i < a.k; i += nwt) {
@@ -805,7 +902,7 @@ cudaError_t launch_idx16_spmspv(const Idx16Args& a, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   if (a.k <= 0) return cudaSuccess;
   const bool fused = a.kidx == nullptr;
-  const size_t smem = fused ? sel_layout(a.I, 0, true).end : 0;
+  const size_t smem = fused ? sel_layout(a.I, 0, a.I).end : 0;
   const int warps = IDX16_THREADS / 32;
   const int grid = (int)std::min<int64_t>((int64_t)dp.nsm * 2, ((int64_t)a.k + warps - 1) / warps);
   if (fused) {
