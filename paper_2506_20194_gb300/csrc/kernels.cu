@@ -689,6 +689,8 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       return mbar_wait_bounded(&full[q.slot], (uint32_t)(q.n & 1), &abort_flag);
     };
     auto release = [&](const SlotCursor& q) { mbar_arrive(&empty[q.slot]); };
+    // The ring can hold every consumer's partial rows for the final flush.
+    const bool scratch_ok = (size_t)nslot * slot_bytes >= (size_t)CMB_NC * SEG_ROWS * sizeof(float);
     int64_t u = u0;
     int piece = 0;
     while (u < u1) {
@@ -756,13 +758,11 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
         if (lane == 0) release(sc);
         sc.advance(CMB_NC, nslot);
       }
-      float* tb = tile + (piece & 1) * SEG_ROWS;
-      if (any) {
-#pragma unroll
-        for (int t = 0; t < 32; ++t) atomicAdd(&tb[32 * lane + ((t + lane) & 31)], acc[t]);
-      }
-      if (piece == 0 && ctid == 0) {
-        // First reduction into y: every CTA must have zeroed its slice.
+      const CmbProb& P = a.p[pc.p];
+      const int rows = min(SEG_ROWS, P.O - pc.s * SEG_ROWS);
+      float* yb = P.y + (size_t)pc.s * SEG_ROWS;
+      // First reduction into y: every CTA must have zeroed its slice.
+      auto wait_grid = [&]() {
         const uint64_t t0 = globaltimer_ns();
         while (ld_acquire_gpu(a.bar + 1) == gen0) {
           __nanosleep(64);
@@ -772,28 +772,63 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
             break;
           }
         }
-      }
-      named_bar_sync(1, CMB_NC * 32);
-      const CmbProb& P = a.p[pc.p];
-      const int rows = min(SEG_ROWS, P.O - pc.s * SEG_ROWS);
-      float* yb = P.y + (size_t)pc.s * SEG_ROWS;
-      for (int g = ctid; 4 * g < rows; g += CMB_NC * 32) {
-        float vv[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int r = 4 * g + e;
-          if (r < rows) {
-            const int ix = tile_index(r);
-            vv[e] = tb[ix];
-            tb[ix] = 0.f;
-          } else {
-            vv[e] = 0.f;
-          }
-        }
+      };
+      auto add_rows = [&](int g, const float (&vv)[4]) {
         if (4 * g + 3 < rows) {
           red_add_v4(yb + 4 * g, vv[0], vv[1], vv[2], vv[3]);
         } else {
           for (int e = 0; e < 4 && 4 * g + e < rows; ++e) atomicAdd(yb + 4 * g + e, vv[e]);
+        }
+      };
+      if (pend == u1 && scratch_ok) {
+        // This CTA's last piece: once every consumer passes the barrier all
+        // items are consumed and no copy is in flight, so the ring is free.
+        // Each consumer stores its partial rows to its own SEG_ROWS floats
+        // of it, then the partials are summed four rows at a time, with no
+        // shared-memory atomics.  Rows 32 L + 4 i .. + 3 sit in 16-byte chunk
+        // (i + L) % 8 of block L, so both the stores and the loads of eight
+        // consecutive lanes hit eight different bank groups.
+        named_bar_sync(1, CMB_NC * 32);
+        float4* mine = reinterpret_cast<float4*>(ring) + (size_t)c * (SEG_ROWS / 4);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          mine[8 * lane + ((i + lane) & 7)] =
+              make_float4(acc[4 * i], acc[4 * i + 1], acc[4 * i + 2], acc[4 * i + 3]);
+        if (piece == 0 && ctid == 0) wait_grid();
+        named_bar_sync(1, CMB_NC * 32);
+        const float4* part = reinterpret_cast<const float4*>(ring);
+        for (int g = ctid; 4 * g < rows; g += CMB_NC * 32) {
+          const int at = 8 * (g >> 3) + (((g & 7) + (g >> 3)) & 7);
+          float vv[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int w = 0; w < CMB_NC; ++w) {
+            const float4 q4 = part[(size_t)w * (SEG_ROWS / 4) + at];
+            vv[0] += q4.x; vv[1] += q4.y; vv[2] += q4.z; vv[3] += q4.w;
+          }
+          add_rows(g, vv);
+        }
+      } else {
+        float* tb = tile + (piece & 1) * SEG_ROWS;
+        if (any) {
+#pragma unroll
+          for (int t = 0; t < 32; ++t) atomicAdd(&tb[32 * lane + ((t + lane) & 31)], acc[t]);
+        }
+        if (piece == 0 && ctid == 0) wait_grid();
+        named_bar_sync(1, CMB_NC * 32);
+        for (int g = ctid; 4 * g < rows; g += CMB_NC * 32) {
+          float vv[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int r = 4 * g + e;
+            if (r < rows) {
+              const int ix = tile_index(r);
+              vv[e] = tb[ix];
+              tb[ix] = 0.f;
+            } else {
+              vv[e] = 0.f;
+            }
+          }
+          add_rows(g, vv);
         }
       }
       ++piece;
