@@ -33,7 +33,7 @@ struct CmbArgs {
   int slot_bytes;        // in: largest record of the launch's weights (bytes);
                          // the launcher rounds it and picks the slot count
   int nslot;             // set by the launcher (a multiple of the consumer count)
-  int group;             // set by the launcher: records a consumer waits for at once
+  int group;             // set by the launcher: records a consumer waits for at once (1 or 2)
   int list_cap;          // set by the launcher: kept-list entries a CTA emits
 };
 

@@ -418,34 +418,6 @@ __device__ __forceinline__ void decode_two(const uint8_t* ra, uint16_t xa, const
   }
 }
 
-// Four records of the same segment at once (two packed prefix sums, four
-// independent load chains per bit position).
-__device__ __forceinline__ void decode_four(const uint8_t* const (&r)[4], const uint16_t (&xv)[4],
-                                            float (&acc)[32], int lane) {
-  uint32_t m[4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) m[i] = reinterpret_cast<const uint32_t*>(r[i])[lane];
-  const uint32_t c01 = (uint32_t)__popc(m[0]) | ((uint32_t)__popc(m[1]) << 16);
-  const uint32_t c23 = (uint32_t)__popc(m[2]) | ((uint32_t)__popc(m[3]) << 16);
-  const uint32_t e01 = warp_inclusive_scan(c01, lane) - c01;
-  const uint32_t e23 = warp_inclusive_scan(c23, lane) - c23;
-  const uint16_t* p[4] = {
-      reinterpret_cast<const uint16_t*>(r[0] + MASK_BYTES) + (e01 & 0xFFFFu),
-      reinterpret_cast<const uint16_t*>(r[1] + MASK_BYTES) + (e01 >> 16),
-      reinterpret_cast<const uint16_t*>(r[2] + MASK_BYTES) + (e23 & 0xFFFFu),
-      reinterpret_cast<const uint16_t*>(r[3] + MASK_BYTES) + (e23 >> 16)};
-#pragma unroll
-  for (int t = 0; t < 32; ++t) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      if (m[i] & (1u << t)) {
-        acc[t] = fma_f16_f32(*p[i], xv[i], acc[t]);
-        ++p[i];
-      }
-    }
-  }
-}
-
 // One consumer warp decodes one record: lane owns rows 32*lane + t.
 __device__ __forceinline__ void decode_record(const uint8_t* rec, uint16_t xb, float (&acc)[32],
                                               int lane) {
@@ -703,33 +675,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       for (int t = 0; t < 32; ++t) acc[t] = 0.f;
       bool any = false;
       int v = va + ((c - va % CMB_NC) % CMB_NC + CMB_NC) % CMB_NC;
-      // this consumer's items four at a time, then in pairs, then alone
-      if (a.group >= 4) {
-        for (; v + 3 * CMB_NC < vb; v += 4 * CMB_NC) {
-          SlotCursor q4[4];
-          bool ok = !abort_flag;
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            q4[i].set(v + i * CMB_NC, nslot);
-            ok = ok && wait_item(q4[i]);
-          }
-          if (ok) {
-            const uint8_t* const rr[4] = {ring + (size_t)q4[0].slot * slot_bytes,
-                                          ring + (size_t)q4[1].slot * slot_bytes,
-                                          ring + (size_t)q4[2].slot * slot_bytes,
-                                          ring + (size_t)q4[3].slot * slot_bytes};
-            const uint16_t xv[4] = {(uint16_t)xval[q4[0].slot], (uint16_t)xval[q4[1].slot],
-                                    (uint16_t)xval[q4[2].slot], (uint16_t)xval[q4[3].slot]};
-            decode_four(rr, xv, acc, lane);
-            any = true;
-          }
-          __syncwarp();
-          if (lane == 0) {
-#pragma unroll
-            for (int i = 0; i < 4; ++i) release(q4[i]);
-          }
-        }
-      }
+      // this consumer's items in pairs, then alone
       SlotCursor sc, sc2;
       sc.set(v, nslot);
       if (a.group >= 2) {
@@ -863,7 +809,7 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   nslot = std::min(nslot, CMB_MAX_SLOTS);
   nslot -= nslot % CMB_NC;
   if (nslot < std::max(32, CMB_NC)) return cudaErrorInvalidValue;
-  a.group = nslot >= 4 * CMB_NC ? 4 : (nslot >= 2 * CMB_NC ? 2 : 1);
+  a.group = nslot >= 2 * CMB_NC ? 2 : 1;   // pairs: waiting for more records costs more than it gains
   a.nslot = nslot;
   a.slot_bytes = slot_bytes;
   const size_t smem = cmb_layout(a.I, fused, a.list_cap, nslot, slot_bytes).total;
