@@ -513,6 +513,7 @@ template <bool FUSED>
 __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArgs a) {
   extern __shared__ __align__(128) uint8_t sm[];
   __shared__ volatile int abort_flag;
+  __shared__ int grid_open;   // 1 once every CTA has zeroed its slice of y
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nslot = a.nslot, slot_bytes = a.slot_bytes;
   const CmbLayout L = cmb_layout(a.I, FUSED, a.list_cap, nslot, slot_bytes);
@@ -532,8 +533,13 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     mbar_init(&empty[i], 1);
   }
   fence_mbar_init();
+  // Generation of the grid barrier before this CTA arrives on it (read here,
+  // before any of this CTA's warps can arrive).
+  unsigned int gen0 = 0;
   if (tid == 0) {
+    gen0 = ld_relaxed_gpu(a.bar + 1);
     abort_flag = 0;
+    grid_open = 0;
     // Warm L2 with this CTA's share of every offset table.
     for (int p = 0; p < a.np; ++p) {
       const size_t bytes = align_up(((size_t)a.I * a.p[p].S + 1) * 4, 16);
@@ -628,6 +634,20 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       }
       if (stop) break;
     }
+    // Every copy is issued: wait here, off the consumers' path, for the grid
+    // barrier, and tell the consumers through shared memory.
+    if (lane == 0) {
+      const uint64_t t0 = globaltimer_ns();
+      while (ld_acquire_gpu(a.bar + 1) == gen0) {
+        __nanosleep(64);
+        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
+          atomicOr(&g_status, STATUS_TIMEOUT);
+          abort_flag = 1;
+          break;
+        }
+      }
+      st_release_cta_shared(&grid_open, 1);
+    }
     if (abort_flag) {
       // Let this lane's copies still in flight land before the CTA exits.
       for (int v = last_v; v >= 0 && v > last_v - nslot; v -= 32) {
@@ -643,9 +663,9 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     // Arrive on the grid barrier once this CTA's slice of y is zero (ordered
     // by the __syncthreads above); done here, off the selection's path, its
     // latency overlaps the first record fetches.
-    unsigned int gen0 = 0;
+    unsigned int gen0c = 0;
     if (ctid == 0) {
-      gen0 = ld_relaxed_gpu(a.bar + 1);
+      gen0c = ld_relaxed_gpu(a.bar + 1);
       if (atom_add_acq_rel_gpu(a.bar, 1u) == gridDim.x - 1) {   // last arriver opens it
         a.bar[0] = 0u;
         red_add_release_gpu(a.bar + 1, 1u);
@@ -707,15 +727,21 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       const CmbProb& P = a.p[pc.p];
       const int rows = min(SEG_ROWS, P.O - pc.s * SEG_ROWS);
       float* yb = P.y + (size_t)pc.s * SEG_ROWS;
-      // First reduction into y: every CTA must have zeroed its slice.
+      // First reduction into y: every CTA must have zeroed its slice.  The
+      // producer, once it has issued every copy, waits for the grid barrier
+      // and sets grid_open; a flush that comes earlier polls the barrier
+      // itself (it must not wait for the producer, which may be waiting for
+      // this flush's consumers to free slots).
       auto wait_grid = [&]() {
+        if (ld_acquire_cta_shared(&grid_open) == 1) return;
         const uint64_t t0 = globaltimer_ns();
-        while (ld_acquire_gpu(a.bar + 1) == gen0) {
+        while (ld_acquire_gpu(a.bar + 1) == gen0c) {
+          if (ld_acquire_cta_shared(&grid_open) == 1) return;
           __nanosleep(64);
           if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
             atomicOr(&g_status, STATUS_TIMEOUT);
             abort_flag = 1;
-            break;
+            return;
           }
         }
       };
