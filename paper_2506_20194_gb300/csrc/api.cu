@@ -311,6 +311,7 @@ static int spmspv_common(const duo_packed* const* hs, int n, const void* x, cons
       a.p[p].y = ys[p];
       a.p[p].O = (int)hs[p]->out;
       a.p[p].S = (int)hs[p]->nseg;
+      a.p[p].dens = (float)((double)hs[p]->nnz / ((double)hs[p]->out * (double)hs[p]->in));
     }
     e = duo::launch_cmb_spmspv(a, st);
     if (e == cudaErrorInvalidValue) return DUO_ERANGE;

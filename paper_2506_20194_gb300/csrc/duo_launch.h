@@ -10,6 +10,7 @@
 namespace duo {
 
 constexpr int kMaxProblems = 4;
+constexpr int kMaxRuns = 128;   // (problem, segment) runs a launch may split by
 constexpr int kSegRows = 1024;
 
 struct CmbProb {
@@ -18,6 +19,7 @@ struct CmbProb {
   float* y;              // fp32[O], zeroed before the launch
   int O;
   int S;
+  float dens;            // non-zeros / (O * I): to estimate record sizes
 };
 
 struct CmbArgs {
@@ -35,6 +37,10 @@ struct CmbArgs {
   int nslot;             // set by the launcher (a multiple of the consumer count)
   int group;             // set by the launcher: records a consumer waits for at once (1 or 2)
   int list_cap;          // set by the launcher: kept-list entries a CTA emits
+  int nruns;             // set by the launcher: > 0 when each (problem, segment)
+                         // run has CTAs of its own: run r (items r*k .. r*k+k-1)
+                         // goes to CTAs run_cta[r] .. run_cta[r+1]-1
+  uint16_t run_cta[kMaxRuns + 1];
 };
 
 struct Idx16Args {

@@ -562,10 +562,19 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       base += a.p[p].O;
     }
   }
-  int64_t total = 0;
-  for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
-  const int64_t u0 = total * blockIdx.x / gridDim.x;
-  const int64_t u1 = total * (blockIdx.x + 1) / gridDim.x;
+  int64_t u0, u1;   // this CTA's items
+  if (a.nruns > 0) {
+    int r = 0;
+    while (r + 1 < a.nruns && (unsigned)a.run_cta[r + 1] <= blockIdx.x) ++r;
+    const int64_t n = a.run_cta[r + 1] - a.run_cta[r], m = blockIdx.x - a.run_cta[r];
+    u0 = (int64_t)r * a.k + (int64_t)a.k * m / n;
+    u1 = (int64_t)r * a.k + (int64_t)a.k * (m + 1) / n;
+  } else {
+    int64_t total = 0;
+    for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
+    u0 = total * blockIdx.x / gridDim.x;
+    u1 = total * (blockIdx.x + 1) / gridDim.x;
+  }
   const int nv = (int)(u1 - u0);
   // This CTA's items use the kept ranks r0, r0 + 1, ... (mod k): only those
   // entries of the kept list are emitted, at positions 0, 1, ...
@@ -820,8 +829,41 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   if (total <= 0) return cudaSuccess;
   const int grid = (int)std::min<int64_t>(dp.nsm, total);
   if ((total + grid - 1) / grid >= (int64_t)1 << 30) return cudaErrorInvalidValue;
+  // Item split.  Items are the (problem, segment) runs of k kept channels
+  // each, in order.  When every run can have CTAs of its own, runs get CTAs in
+  // proportion to their estimated bytes (record = mask + 2 bytes per expected
+  // non-zero) and no CTA spans two runs: a run boundary inside a CTA would
+  // cost a mid-stream flush of all its consumers' rows.  Otherwise the items
+  // are split evenly.
+  int nruns = 0;
+  for (int p = 0; p < a.np; ++p) nruns += a.p[p].S;
+  int64_t per_cta = (total + grid - 1) / grid;
+  a.nruns = 0;
+  if (nruns <= kMaxRuns && nruns <= grid) {
+    double w[kMaxRuns];
+    int n[kMaxRuns];
+    int r = 0;
+    for (int p = 0; p < a.np; ++p)
+      for (int s = 0; s < a.p[p].S; ++s, ++r) {
+        const int rows = std::min(SEG_ROWS, a.p[p].O - s * SEG_ROWS);
+        w[r] = (double)MASK_BYTES + 2.0 * (double)a.p[p].dens * rows;
+        n[r] = 1;
+      }
+    for (int extra = grid - nruns; extra > 0; --extra) {
+      int best = 0;
+      for (int q = 1; q < nruns; ++q)
+        if (w[q] * n[best] > w[best] * n[q]) best = q;
+      ++n[best];
+    }
+    a.run_cta[0] = 0;
+    per_cta = 0;
+    for (int q = 0; q < nruns; ++q) {
+      a.run_cta[q + 1] = (uint16_t)(a.run_cta[q] + n[q]);
+      per_cta = std::max<int64_t>(per_cta, (a.k + n[q] - 1) / n[q]);
+    }
+    a.nruns = nruns;
+  }
   // Kept-list window of a CTA: at most its item count, at most k.
-  const int64_t per_cta = (total + grid - 1) / grid;
   a.list_cap = fused ? (int)std::min<int64_t>(per_cta, a.k) : 0;
   // Slot size: the largest record among the launch's weights (given by the
   // caller in a.slot_bytes); slot count: as many as the shared memory holds,
