@@ -180,6 +180,15 @@ __device__ __forceinline__ bool wait_shared_eq(const int* p, int want, volatile 
   }
 }
 
+// Programmatic dependent launch: wait until the previous kernel of the
+// stream has completed and its memory is visible (returns at once when the
+// launch has no programmatic dependency), and let the next kernel of the
+// stream be scheduled as soon as this grid's CTAs leave their SMs.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }

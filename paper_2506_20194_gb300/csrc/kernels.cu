@@ -526,21 +526,20 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   uint16_t* klist = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.klist) : nullptr;
   SelShared* sel = FUSED ? reinterpret_cast<SelShared*>(sm + L.sel.sel) : nullptr;
 
-  // ---- prologue: x, mbarriers, tile, this CTA's slice of y = 0 ----
-  if (FUSED) load_x_to_smem(xs, a.x, a.I);   // issued first: its latency overlaps the rest
+  // ---- prologue ----
+  // Work that touches nothing the previous kernel of the stream may write
+  // runs before griddep_wait(), overlapping that kernel's last CTAs: ring
+  // mbarriers, shared-memory state, and an L2 warm-up of this CTA's share of
+  // every offset table (a hint only).
+  griddep_launch_dependents();
   for (int i = tid; i < nslot; i += CMB_THREADS) {
     mbar_init(&full[i], 1);
     mbar_init(&empty[i], 1);
   }
   fence_mbar_init();
-  // Generation of the grid barrier before this CTA arrives on it (read here,
-  // before any of this CTA's warps can arrive).
-  unsigned int gen0 = 0;
   if (tid == 0) {
-    gen0 = ld_relaxed_gpu(a.bar + 1);
     abort_flag = 0;
     grid_open = 0;
-    // Warm L2 with this CTA's share of every offset table.
     for (int p = 0; p < a.np; ++p) {
       const size_t bytes = align_up(((size_t)a.I * a.p[p].S + 1) * 4, 16);
       const size_t lo = align_up(bytes * blockIdx.x / gridDim.x, 16);
@@ -550,6 +549,15 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   }
   for (int i = tid; i < 2 * SEG_ROWS; i += CMB_THREADS) tile[i] = 0.f;
   if (FUSED) select_clear(sel);
+  // Inputs, y and the grid barrier words may be the previous kernel's.
+  griddep_wait();
+  if (FUSED) load_x_to_smem(xs, a.x, a.I);
+  // Generation of the grid barrier before this CTA arrives on it (read here,
+  // before any of this CTA's warps can arrive).
+  unsigned int gen0 = 0;
+  if (tid == 0) {
+    gen0 = ld_relaxed_gpu(a.bar + 1);
+  }
   {
     int64_t ytot = 0;
     for (int p = 0; p < a.np; ++p) ytot += a.p[p].O;
@@ -889,11 +897,17 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   cfg.blockDim = dim3(CMB_THREADS);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  // Cooperative: all CTAs are co-resident (the in-kernel grid barrier).
+  // Programmatic stream serialization: this launch may start while the
+  // previous kernel of the stream finishes; the kernel waits for it
+  // (griddepcontrol.wait) before it reads its inputs or writes y.
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeCooperative;
   attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   e = cudaLaunchKernelEx(&cfg, kern, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
