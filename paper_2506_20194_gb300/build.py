@@ -30,8 +30,11 @@ def nvcc_path() -> str:
 
 def _compile(src: str, extra: list[str]) -> str:
     obj = os.path.join(BUILD_DIR, os.path.splitext(src)[0] + ".o")
-    cmd = [nvcc_path(), *ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
-           "-I", os.path.join(ROOT, "include"), "-c", os.path.join(CSRC, src), "-o", obj, *extra]
+    # Warnings are errors: a host-only call from __host__ __device__ code, for
+    # one, is only a warning but leaves the device code undefined.
+    cmd = [nvcc_path(), *ARCH, "-O3", "-lineinfo", "-std=c++17", "-Werror", "all-warnings",
+           "-Xcompiler", "-fPIC", "-I", os.path.join(ROOT, "include"), "-c", os.path.join(CSRC, src),
+           "-o", obj, *extra]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
