@@ -36,8 +36,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch of
 # the fused kernel from one ncu capture, valid only for the kernel source it
 # was taken on (sha256 of kernels.cu + duo_device.cuh, first 16 hex digits).
-TRAFFIC = {"sha": "5b61f86e724d73b1",
-           "per_launch_bytes": [29114624.0, 9760000.0, 51926528.0, 26107136.0]}
+TRAFFIC = {"sha": "485b3751699d2b20",
+           "per_launch_bytes": [29127680.0, 9773312.0, 51913984.0, 26120960.0]}
 
 
 def parse():
