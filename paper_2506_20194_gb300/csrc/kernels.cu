@@ -597,7 +597,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
 
   if (warp == 0) {
     // ---------------- producer ----------------
-    constexpr int PQ = 8;
+    constexpr int PQ = 2;   // rounds queued ahead: deeper queues only add code and start-up work
     const uint64_t pol = policy_evict_first();
     int last_v = -1;
     bool stop = false;
