@@ -437,17 +437,17 @@ __device__ __forceinline__ void decode_record(const uint8_t* rec, uint16_t xb, f
 // Item cursor: (product p, segment s, kept rank i) of a linear item index.
 struct ItemCursor {
   int p, s, i;
-  __device__ __forceinline__ void set(const CmbArgs& a, int64_t u) {
-    const int64_t k = a.k;
-    int64_t base = 0;
+  __device__ __forceinline__ void set(const CmbArgs& a, uint32_t u) {   // item counts < 2^31
+    const uint32_t k = (uint32_t)a.k;
+    uint32_t base = 0;
     p = 0;
-    while (p < a.np - 1 && u >= base + (int64_t)a.p[p].S * k) {
-      base += (int64_t)a.p[p].S * k;
+    while (p < a.np - 1 && u >= base + (uint32_t)a.p[p].S * k) {
+      base += (uint32_t)a.p[p].S * k;
       ++p;
     }
-    const int64_t rem = u - base;
+    const uint32_t rem = u - base;
     s = (int)(rem / k);
-    i = (int)(rem - (int64_t)s * k);
+    i = (int)(rem - (uint32_t)s * k);
   }
   __device__ __forceinline__ void advance(const CmbArgs& a, int n) {
     i += n;
@@ -558,40 +558,30 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   if (tid == 0) {
     gen0 = ld_relaxed_gpu(a.bar + 1);
   }
-  {
-    int64_t ytot = 0;
-    for (int p = 0; p < a.np; ++p) ytot += a.p[p].O;
-    const int64_t z0 = ytot * blockIdx.x / gridDim.x, z1 = ytot * (blockIdx.x + 1) / gridDim.x;
-    int64_t base = 0;
-    for (int p = 0; p < a.np; ++p) {
-      const int64_t lo = z0 > base ? z0 : base;
-      const int64_t hi = z1 < base + a.p[p].O ? z1 : base + a.p[p].O;
-      for (int64_t r = lo + tid; r < hi; r += CMB_THREADS) a.p[p].y[r - base] = 0.f;
-      base += a.p[p].O;
-    }
-  }
-  int64_t u0, u1;   // this CTA's items
+  uint32_t u0, u1;   // this CTA's items (32-bit: the launcher keeps counts < 2^31)
+  int r0 = 0;        // kept rank of its first item
   if (a.nruns > 0) {
     int r = 0;
     while (r + 1 < a.nruns && (unsigned)a.run_cta[r + 1] <= blockIdx.x) ++r;
-    const int64_t n = a.run_cta[r + 1] - a.run_cta[r], m = blockIdx.x - a.run_cta[r];
-    u0 = (int64_t)r * a.k + (int64_t)a.k * m / n;
-    u1 = (int64_t)r * a.k + (int64_t)a.k * (m + 1) / n;
+    const uint32_t n = a.run_cta[r + 1] - a.run_cta[r], m = blockIdx.x - a.run_cta[r];
+    const uint32_t k = (uint32_t)a.k;   // k * m < 2^32: k <= 65535, m < 1024
+    u0 = (uint32_t)r * k + k * m / n;
+    u1 = (uint32_t)r * k + k * (m + 1) / n;
+    r0 = (int)(k * m / n);
   } else {
-    int64_t total = 0;
-    for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
-    u0 = total * blockIdx.x / gridDim.x;
-    u1 = total * (blockIdx.x + 1) / gridDim.x;
+    uint32_t total = 0;
+    for (int p = 0; p < a.np; ++p) total += (uint32_t)a.p[p].S * (uint32_t)a.k;
+    u0 = (uint32_t)((uint64_t)total * blockIdx.x / gridDim.x);
+    u1 = (uint32_t)((uint64_t)total * (blockIdx.x + 1) / gridDim.x);
+    if (FUSED) {
+      ItemCursor first;
+      first.set(a, u0);
+      r0 = first.i;
+    }
   }
   const int nv = (int)(u1 - u0);
-  // This CTA's items use the kept ranks r0, r0 + 1, ... (mod k): only those
+  // The CTA's items use the kept ranks r0, r0 + 1, ... (mod k): only those
   // entries of the kept list are emitted, at positions 0, 1, ...
-  int r0 = 0;
-  if (FUSED) {
-    ItemCursor first;
-    first.set(a, u0);
-    r0 = first.i;
-  }
   __syncthreads();
   if (FUSED) select_topk(xs, a.I, a.k, (uint32_t)r0, (uint32_t)a.list_cap, klist, nullptr, sel);
 
@@ -677,9 +667,23 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     // ---------------- consumers ----------------
     const int c = warp - 1;
     const int ctid = tid - 32;
-    // Arrive on the grid barrier once this CTA's slice of y is zero (ordered
-    // by the __syncthreads above); done here, off the selection's path, its
-    // latency overlaps the first record fetches.
+    // Zero this CTA's slice of the outputs and arrive on the grid barrier:
+    // done here, off the selection's path, while the first records are in
+    // flight.  The named barrier orders every consumer's stores before
+    // consumer 0's release.
+    {
+      int64_t ytot = 0;
+      for (int p = 0; p < a.np; ++p) ytot += a.p[p].O;
+      const int64_t z0 = ytot * blockIdx.x / gridDim.x, z1 = ytot * (blockIdx.x + 1) / gridDim.x;
+      int64_t base = 0;
+      for (int p = 0; p < a.np; ++p) {
+        const int64_t lo = z0 > base ? z0 : base;
+        const int64_t hi = z1 < base + a.p[p].O ? z1 : base + a.p[p].O;
+        for (int64_t r = lo + ctid; r < hi; r += CMB_NC * 32) a.p[p].y[r - base] = 0.f;
+        base += a.p[p].O;
+      }
+    }
+    named_bar_sync(1, CMB_NC * 32);
     unsigned int gen0c = 0;
     if (ctid == 0) {
       gen0c = ld_relaxed_gpu(a.bar + 1);
@@ -700,13 +704,13 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     auto release = [&](const SlotCursor& q) { mbar_arrive(&empty[q.slot]); };
     // The ring can hold every consumer's partial rows for the final flush.
     const bool scratch_ok = (size_t)nslot * slot_bytes >= (size_t)CMB_NC * SEG_ROWS * sizeof(float);
-    int64_t u = u0;
+    uint32_t u = u0;
     int piece = 0;
     while (u < u1) {
       ItemCursor pc;
       pc.set(a, u);
-      const int64_t seg_end = u + (a.k - pc.i);   // end of this (p, s) run
-      const int64_t pend = seg_end < u1 ? seg_end : u1;
+      const uint32_t seg_end = u + (uint32_t)(a.k - pc.i);   // end of this (p, s) run
+      const uint32_t pend = seg_end < u1 ? seg_end : u1;
       const int va = (int)(u - u0), vb = (int)(pend - u0);
 #pragma unroll
       for (int t = 0; t < 32; ++t) acc[t] = 0.f;
@@ -835,6 +839,7 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   int64_t total = 0;
   for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
   if (total <= 0) return cudaSuccess;
+  if (total >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;   // item indices are 32-bit
   const int grid = (int)std::min<int64_t>(dp.nsm, total);
   if ((total + grid - 1) / grid >= (int64_t)1 << 30) return cudaErrorInvalidValue;
   // Item split.  Items are the (problem, segment) runs of k kept channels
