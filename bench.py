@@ -53,6 +53,11 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--profile", action="store_true",
                     help="small case for ncu: 2 layers, a few direct (ungraphed) layer steps")
+    ap.add_argument("--stack", default=None,
+                    choices=("llama2-7b-layer", "llama3-8b-stack", "llama2-13b-stack", "llama2-70b-stack"),
+                    help="per-token time over every layer of a stack workload (one CUDA graph per token)")
+    ap.add_argument("--stack-layers", type=int, default=None, help="layers of the stack (default: all)")
+    ap.add_argument("--stack-pw", type=float, default=None, help="weight sparsity (default: the workload's)")
     return ap.parse_args()
 
 
@@ -521,10 +526,75 @@ def run_profile(args):
     print("profile workload done", flush=True)
 
 
+def run_stack(args):
+    """Per-token time of a whole stack: every layer's four launches (q/k/v,
+    o, gate/up, down) in one CUDA graph, each layer with its own packed
+    weights and inputs (no rotation needed: a 32-80 layer stack is far above
+    L2).  Prints one JSON line; not the default bench line."""
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2506_20194_gb300 import duo, synth
+    duo.load_library()
+    wl = synth.WORKLOADS[args.stack]
+    shape = wl["shape"]
+    L = args.stack_layers or wl["layers"]
+    pw = wl["pw"] if args.stack_pw is None else args.stack_pw
+    px = args.px
+    ys = {p: torch.empty(shape.O(p), dtype=torch.float32, device=dev) for p in synth.PROJS}
+    layers, breq, packed = [], 0.0, 0
+    t0 = time.time()
+    for l in range(L):
+        hs, nnz = {}, {}
+        for p in synth.PROJS:
+            W = synth.layer_weight(wl, p, layer=l, device=dev, pw=pw)
+            hs[p] = duo.duo_pack(W, "bitmask")
+            nnz[p] = (W != 0).sum(dim=0).to(torch.int64)
+            packed += hs[p].query().data_bytes + hs[p].query().index_bytes
+            del W
+        xs = {s: synth.layer_input(wl, s, layer=l, device=dev) for s in STAGE_SRC}
+        lay = dict(h=hs, nnz=nnz, x=xs, y=ys)
+        breq += required_bytes_layer(duo, shape, lay, px)[0]
+        del lay["nnz"]
+        layers.append(lay)
+    torch.cuda.synchronize()
+    pack_s = time.time() - t0
+
+    def fn():
+        for lay in layers:
+            for si in range(len(STAGES)):
+                stage_call(duo, shape, lay, px, si)
+    g = capture(fn)
+    time_graph(g, max(3, args.warmup if args.warmup < 50 else 5))
+    reps = max(5, min(args.steps, 200))
+    sampler = ClockSampler(0)
+    sampler.start()
+    t = time_graph(g, reps)
+    clocks = sampler.stop()
+    assert duo.duo_device_status() == duo.DUO_OK
+    us_token = t / reps * 1e6
+    peak, peak_kind = peaks()
+    gbs = breq / (us_token * 1e-6) / 1e9
+    dense_bytes = 2.0 * L * sum(shape.O(p) * shape.I(p) for p in synth.PROJS)
+    line = {"metric": "per-token µs over the stack (batch-1 dual-sparse spMspV, every projection of every layer)",
+            "value": us_token, "unit": "us/token", "higher_is_better": False,
+            "workload": args.stack, "layers": L, "pw": pw, "px": px,
+            "required_GB_per_token": breq / 1e9, "GB/s": gbs, "frac_of_peak": gbs / peak, "peak": peak,
+            "peak_kind": peak_kind, "roofline_us_per_token": breq / (peak * 1e9) * 1e6,
+            "dense_fp16_GB_per_token": dense_bytes / 1e9,
+            "dense_roofline_us_per_token": dense_bytes / (peak * 1e9) * 1e6,
+            "packed_GB": packed / 1e9, "pack_seconds": pack_s, "launches_per_token": 4 * L,
+            "reps": reps, "clocks": clocks, "data": "synthetic", "dtype": "f16"}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     if args.profile:
         run_profile(args)
+    elif args.stack is not None:
+        run_stack(args)
     elif args.impl == "reference":
         run_reference(args)
     else:
