@@ -17,6 +17,8 @@ from .duo_oracle import (  # noqa: F401
     IDX16_MAGIC,
     k_from_pct,
     oracle_sparsify,
+    oracle_sparsify_threshold,
+    oracle_spmspv_threshold,
     oracle_spmspv,
     oracle_spmspv_rows,
     exact_spmspv_rows_scaled,

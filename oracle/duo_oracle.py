@@ -25,6 +25,9 @@ Readings taken where the paper is silent (each is listed in the design doc):
   * the oracle requires x to be NaN-free (the CUDA path orders NaN above Inf
     by bit pattern; the paper does not define either);
   * a weight entry is pruned iff it compares equal to zero (+0 or -0);
+  * the threshold mask (§5's threshold-based activation sparsity) keeps
+    |x_j| > |tau| strictly, as the thresholding function it cites zeroes
+    entries at or below the threshold;
   * y is accumulated and returned in fp64 here (fp32 on the GPU).
 """
 from __future__ import annotations
@@ -84,6 +87,39 @@ def oracle_sparsify(x16, k: int):
     order = np.lexsort((j, -a))          # by |x| descending, then j ascending
     K = np.sort(order[:k])
     return K.astype(np.uint16), x[K].copy()
+
+
+def oracle_sparsify_threshold(x16, tau):
+    """Threshold activation mask (§5, compatibility with threshold-based
+    activation sparsity, Table 3(b)): instead of the k largest magnitudes,
+    the mask keeps every channel whose magnitude exceeds a threshold fixed
+    beforehand for the layer.  Entries with |x_j| <= |tau| are dropped, so the
+    comparison is strict; the sign of ``tau`` is ignored.
+
+    Returns ``(kept_idx, kept_val)``: the kept channel ids in ASCENDING order
+    as uint16 and the unchanged fp16 values x[kept_idx].  The number kept
+    depends on x.
+    """
+    x = _as_f16(x16).reshape(-1)
+    I = x.shape[0]
+    if I > 65535:
+        raise ValueError("channel ids are uint16: I must be <= 65535")
+    a = np.abs(x.astype(np.float64))
+    t = abs(float(np.float16(tau)))
+    if np.isnan(a).any() or math.isnan(t):
+        raise ValueError("the oracle defines the kept set for NaN-free x and tau only")
+    K = np.nonzero(a > t)[0]
+    return K.astype(np.uint16), x[K].copy()
+
+
+def oracle_spmspv_threshold(W16, x16, tau) -> np.ndarray:
+    """y = W (x ⊙ m^x) in fp64 (§3) with the threshold mask of
+    :func:`oracle_sparsify_threshold`."""
+    W = _as_f16(W16)
+    if W.ndim != 2 or W.shape[1] != _as_f16(x16).size:
+        raise ValueError("W must be O x I with I = len(x)")
+    K, xv = oracle_sparsify_threshold(x16, tau)
+    return W[:, K.astype(np.int64)].astype(np.float64) @ xv.astype(np.float64)
 
 
 def oracle_spmspv(W16, x16, k: int) -> np.ndarray:

@@ -57,6 +57,12 @@ def _parse_golden():
                 K = [int(t) for t in tok[3:yi]]
                 y = [float(t) for t in tok[yi + 1:]]
                 cases.append((k, K, y))
+            elif tok[0] == "thresh":
+                tau = float(tok[1].split("=")[1])
+                yi = tok.index("y")
+                K = [int(t) for t in tok[3:yi]]
+                y = [float(t) for t in tok[yi + 1:]]
+                cases.append(("tau", tau, K, y))
             elif tok[0] == "cmb_record":
                 j = int(tok[1].split("=")[1])
                 word0 = int(tok[3])
@@ -68,11 +74,62 @@ def _parse_golden():
 
 def test_golden_hand_worked_example():
     W, x, cases, _ = _parse_golden()
-    for k, K, y in cases:
+    for case in cases:
+        if case[0] == "tau":
+            continue
+        k, K, y = case
         Kc, vals = orc.oracle_sparsify(x, k)
         assert list(Kc) == K
         assert np.array_equal(vals.view(np.uint16), x[K].view(np.uint16))
         assert np.array_equal(orc.oracle_spmspv(W, x, k), np.array(y))
+
+
+def test_golden_threshold_cases():
+    W, x, cases, _ = _parse_golden()
+    tcases = [c for c in cases if c[0] == "tau"]
+    assert len(tcases) == 5
+    for _, tau, K, y in tcases:
+        Kc, vals = orc.oracle_sparsify_threshold(x, tau)
+        assert list(Kc) == K
+        assert np.array_equal(vals.view(np.uint16), x[K].view(np.uint16))
+        assert np.array_equal(orc.oracle_spmspv_threshold(W, x, tau), np.array(y))
+        assert np.array_equal(orc.oracle_spmspv_threshold(W, x, -tau), np.array(y))   # sign ignored
+
+
+def test_threshold_equals_topk_between_magnitudes():
+    """Two independent definitions agree: with no tie at the boundary, the
+    channels above the (k+1)-th largest magnitude are the top-k set."""
+    rng = np.random.default_rng(11)
+    for trial in range(200):
+        I = int(rng.integers(2, 300))
+        x = rng.laplace(size=I).astype(np.float16)
+        a = np.sort(np.abs(x.astype(np.float64)))[::-1]
+        k = int(rng.integers(0, I))
+        if k > 0 and a[k - 1] == a[k]:
+            continue   # tie at the boundary: top-k breaks it by index, a threshold cannot
+        Kt, _ = orc.oracle_sparsify_threshold(x, a[k])
+        Kk, _ = orc.oracle_sparsify(x, k)
+        assert np.array_equal(Kt, Kk)
+
+
+def test_threshold_special_cases():
+    x = np.array([0.0, -0.0, 1.5, -3.0, 0.0, 2.0, -1.5, 65504.0], dtype=np.float16)
+    assert list(orc.oracle_sparsify_threshold(x, 0.0)[0]) == [2, 3, 5, 6, 7]   # the non-zeros
+    assert list(orc.oracle_sparsify_threshold(x, 1.5)[0]) == [3, 5, 7]          # strict
+    assert len(orc.oracle_sparsify_threshold(x, 65504.0)[0]) == 0
+    assert len(orc.oracle_sparsify_threshold(x, np.inf)[0]) == 0
+    inf_x = np.array([np.inf, -np.inf, 1.0], dtype=np.float16)
+    assert list(orc.oracle_sparsify_threshold(inf_x, 65504.0)[0]) == [0, 1]
+    with pytest.raises(ValueError):
+        orc.oracle_sparsify_threshold(np.array([np.nan, 1.0], dtype=np.float16), 0.5)
+    # nested: a larger threshold keeps a subset
+    rng = np.random.default_rng(5)
+    xr = rng.laplace(size=500).astype(np.float16)
+    prev = set(range(500))
+    for tau in (0.0, 0.1, 0.5, 1.0, 2.0, 4.0):
+        cur = set(int(j) for j in orc.oracle_sparsify_threshold(xr, tau)[0])
+        assert cur <= prev
+        prev = cur
 
 
 def test_golden_cmb_records():
