@@ -141,6 +141,40 @@ int duo_spmspv_multi(const duo_packed* const* hs, int n, const void* x_fp16_dev,
                      const uint16_t* kept_idx_dev, const void* kept_val_fp16_dev,
                      int64_t k, float* const* ys_dev, void* stream);
 
+/*
+ * Threshold mask (§5, "compatibility with threshold-based activation
+ * sparsity", Table 3(b)): instead of the k largest magnitudes, keep every
+ * channel whose magnitude is strictly above a threshold fixed beforehand for
+ * the layer (calibrated offline for a target sparsity); the number kept then
+ * depends on x.  tau_fp16 is the threshold as fp16 bits; its sign is ignored
+ * (channel j is kept iff (x_j bits & 0x7FFF) > (tau bits & 0x7FFF), i.e.
+ * |x_j| > |tau| for non-NaN values).
+ *
+ * duo_sparsify_threshold -- the kept channels, ascending.  Async.
+ *   x_fp16_dev        : device, fp16[in], 1 <= in <= 65535.
+ *   kept_idx_dev      : device, uint16[in]: room for every channel; the
+ *                       first *count_dev entries are written.
+ *   kept_val_fp16_dev : device, fp16[in]: x at those ids, bit-exact.
+ *   count_dev         : device, int32: the number kept.
+ * Errors: DUO_EINVAL (NULL, size, alignment), DUO_ECUDA.
+ */
+int duo_sparsify_threshold(const void* x_fp16_dev, int64_t in, uint16_t tau_fp16,
+                           uint16_t* kept_idx_dev, void* kept_val_fp16_dev, int32_t* count_dev,
+                           void* stream);
+
+/*
+ * duo_spmspv_threshold -- y_p = W_p (x ⊙ m^x) for n (1..4) DUO_FMT_BITMASK
+ * handles with the same I, with the threshold mask above computed inside
+ * the launch (each CTA takes a channel range of one (product, segment) run
+ * and keeps the channels above the threshold in it: no ranking across the
+ * vector).  ys_dev[p]: device fp32[O_p], 16-byte aligned, fully overwritten.
+ * Async; same ordering rule as duo_spmspv for calls sharing a first handle.
+ * Errors: DUO_EINVAL, DUO_EFORMAT (not BITMASK), DUO_ERANGE (more (product,
+ * segment) runs than SMs), DUO_ECUDA.
+ */
+int duo_spmspv_threshold(const duo_packed* const* hs, int n, const void* x_fp16_dev,
+                         uint16_t tau_fp16, float* const* ys_dev, void* stream);
+
 /* duo_free -- release a handle and its device memory.  NULL is a no-op
  * (DUO_OK); a handle that is not live (already freed, never created)
  * returns DUO_EINVAL without touching memory.  Synchronises the device

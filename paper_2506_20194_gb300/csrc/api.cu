@@ -261,6 +261,63 @@ int duo_sparsify(const void* x_fp16_dev, int64_t in, int64_t k, uint16_t* kept_i
   return map_err(e);
 }
 
+int duo_sparsify_threshold(const void* x_fp16_dev, int64_t in, uint16_t tau_fp16,
+                           uint16_t* kept_idx_dev, void* kept_val_fp16_dev, int32_t* count_dev,
+                           void* stream) {
+  if (x_fp16_dev == nullptr || kept_idx_dev == nullptr || kept_val_fp16_dev == nullptr ||
+      count_dev == nullptr)
+    return DUO_EINVAL;
+  if (in < 1 || in > 65535) return DUO_EINVAL;
+  if (!aligned(x_fp16_dev, 2) || !aligned(kept_idx_dev, 2) || !aligned(kept_val_fp16_dev, 2) ||
+      !aligned(count_dev, 4))
+    return DUO_EINVAL;
+  int rc = cuda_ready();
+  if (rc != DUO_OK) return rc;
+  cudaError_t e = duo::launch_sparsify_threshold(static_cast<const uint16_t*>(x_fp16_dev), (int)in,
+                                                 tau_fp16, kept_idx_dev,
+                                                 static_cast<uint16_t*>(kept_val_fp16_dev),
+                                                 count_dev, static_cast<cudaStream_t>(stream));
+  return map_err(e);
+}
+
+int duo_spmspv_threshold(const duo_packed* const* hs, int n, const void* x_fp16_dev,
+                         uint16_t tau_fp16, float* const* ys_dev, void* stream) {
+  if (hs == nullptr || ys_dev == nullptr || x_fp16_dev == nullptr) return DUO_EINVAL;
+  if (n < 1 || n > duo::kMaxProblems) return DUO_EINVAL;
+  if (!aligned(x_fp16_dev, 2)) return DUO_EINVAL;
+  for (int p = 0; p < n; ++p) {
+    if (hs[p] == nullptr || ys_dev[p] == nullptr || !aligned(ys_dev[p], 16)) return DUO_EINVAL;
+    if (!is_live(hs[p])) return DUO_EINVAL;
+    if (hs[p]->fmt != DUO_FMT_BITMASK) return DUO_EFORMAT;
+    if (hs[p]->in != hs[0]->in) return DUO_EINVAL;
+  }
+  int rc = cuda_ready();
+  if (rc != DUO_OK) return rc;
+  duo::CmbArgs a{};
+  a.np = n;
+  a.I = (int)hs[0]->in;
+  a.k = 0;   // the launcher sets a cursor bound; the kept count is per CTA
+  a.x = static_cast<const uint16_t*>(x_fp16_dev);
+  a.kidx = nullptr;
+  a.kval = nullptr;
+  a.thresh = 1;
+  a.tau_key = tau_fp16 & 0x7FFFu;
+  a.bar = hs[0]->sync;
+  a.slot_bytes = 0;
+  for (int p = 0; p < n; ++p) {
+    a.slot_bytes = hs[p]->max_record > a.slot_bytes ? hs[p]->max_record : a.slot_bytes;
+    a.p[p].data = static_cast<const uint8_t*>(hs[p]->data);
+    a.p[p].off = static_cast<const uint32_t*>(hs[p]->index);
+    a.p[p].y = ys_dev[p];
+    a.p[p].O = (int)hs[p]->out;
+    a.p[p].S = (int)hs[p]->nseg;
+    a.p[p].dens = (float)((double)hs[p]->nnz / ((double)hs[p]->out * (double)hs[p]->in));
+  }
+  cudaError_t e = duo::launch_cmb_spmspv(a, static_cast<cudaStream_t>(stream));
+  if (e == cudaErrorInvalidValue) return DUO_ERANGE;
+  return map_err(e);
+}
+
 static int spmspv_common(const duo_packed* const* hs, int n, const void* x, const uint16_t* kidx,
                          const void* kval, int64_t k, float* const* ys, void* stream) {
   if (hs == nullptr || ys == nullptr || n < 1 || n > duo::kMaxProblems) return DUO_EINVAL;

@@ -528,4 +528,41 @@ __device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t r0
   __syncthreads();
 }
 
+// Threshold mask (§5, threshold-based activation sparsity): writes the
+// channels j in [c0, c1) with key_j > T in ascending order to klist[0..n) (and
+// their fp16 bits to kvals if given) and returns n to every thread.  Warps
+// take contiguous runs of the range's 32-channel words (lane = channel): one
+// ballot pass counts, a block barrier and a sum over lower warps place each
+// warp's run, a second pass writes.  wcnt needs one entry per warp.  All
+// threads take part; it ends with a __syncthreads.
+__device__ inline int thresh_compact(const uint16_t* xs, int c0, int c1, uint32_t T, uint16_t* klist,
+                                     uint16_t* kvals, uint32_t* wcnt) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  const int wb = c0 >> 5, nwd = c1 > c0 ? ((c1 + 31) >> 5) - wb : 0;
+  const int per = (nwd + nwarps - 1) / nwarps;
+  const int w0 = wb + min(nwd, wid * per), w1 = wb + min(nwd, wid * per + per);
+  auto kept = [&](int j) { return j >= c0 && j < c1 && key_of(xs, j) > T; };
+  uint32_t cnt = 0;
+  for (int w = w0; w < w1; ++w) cnt += (uint32_t)__popc(__ballot_sync(FULL_MASK, kept(32 * w + lane)));
+  if (lane == 0) wcnt[wid] = cnt;
+  __syncthreads();
+  const uint32_t c = lane < nwarps ? wcnt[lane] : 0u;
+  uint32_t base = __reduce_add_sync(FULL_MASK, lane < wid ? c : 0u);
+  const uint32_t total = __reduce_add_sync(FULL_MASK, c);
+  const uint32_t lt = (1u << lane) - 1u;
+  for (int w = w0; w < w1; ++w) {
+    const int j = 32 * w + lane;
+    const bool keep = kept(j);
+    const uint32_t m = __ballot_sync(FULL_MASK, keep);
+    if (keep) {
+      const uint32_t pos = base + (uint32_t)__popc(m & lt);
+      klist[pos] = (uint16_t)j;
+      if (kvals != nullptr) kvals[pos] = xs[j];
+    }
+    base += (uint32_t)__popc(m);
+  }
+  __syncthreads();
+  return (int)total;
+}
+
 }  // namespace duo

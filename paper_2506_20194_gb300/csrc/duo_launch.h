@@ -11,6 +11,10 @@ namespace duo {
 
 constexpr int kMaxProblems = 4;
 constexpr int kMaxRuns = 128;   // (problem, segment) runs a launch may split by
+// Modes of the fused bitmask kernel.
+constexpr int CMB_LISTED = 0;   // kept list given by the caller
+constexpr int CMB_TOPK = 1;     // exact top-k selection in the kernel
+constexpr int CMB_THRESH = 2;   // threshold mask in the kernel
 constexpr int kSegRows = 1024;
 
 struct CmbProb {
@@ -37,6 +41,8 @@ struct CmbArgs {
   int nslot;             // set by the launcher (a multiple of the consumer count)
   int group;             // set by the launcher: records a consumer waits for at once (1 or 2)
   int list_cap;          // set by the launcher: kept-list entries a CTA emits
+  int thresh;            // in: 1 = threshold mask (keep key > tau_key), 0 = top-k / listed
+  uint32_t tau_key;      // in: threshold as an fp16 magnitude bit pattern (bits & 0x7FFF)
   int nruns;             // set by the launcher: > 0 when each (problem, segment)
                          // run has CTAs of its own: run r (items r*k .. r*k+k-1)
                          // goes to CTAs run_cta[r] .. run_cta[r+1]-1
@@ -62,6 +68,8 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a, cudaStream_t st);
 // spMspV over the index format (fused when a.kidx == nullptr).
 cudaError_t launch_idx16_spmspv(const Idx16Args& a, cudaStream_t st);
 // Exact top-k sparsifier: kept ids ascending + their values.
+cudaError_t launch_sparsify_threshold(const uint16_t* x, int I, uint32_t tau_key, uint16_t* kidx,
+                                      uint16_t* kval, int* count, cudaStream_t st);
 cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uint16_t* kval,
                             cudaStream_t st);
 

@@ -331,6 +331,30 @@ cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uin
   return cudaGetLastError();
 }
 
+// Threshold mask alone (parity and standalone use): one CTA.
+__global__ void __launch_bounds__(SPARSIFY_THREADS) sparsify_threshold_kernel(
+    const uint16_t* __restrict__ x, int I, uint32_t T, uint16_t* __restrict__ kidx,
+    uint16_t* __restrict__ kval, int* __restrict__ count) {
+  extern __shared__ __align__(128) uint8_t sm[];
+  const SelLayout L = sel_layout(I, 0, 0);
+  uint16_t* xs = reinterpret_cast<uint16_t*>(sm + L.xs);
+  SelShared* sel = reinterpret_cast<SelShared*>(sm + L.sel);
+  load_x_to_smem(xs, x, I);
+  __syncthreads();
+  const int n = thresh_compact(xs, 0, I, T, kidx, kval, sel->wgt);
+  if (threadIdx.x == 0) *count = n;
+}
+
+cudaError_t launch_sparsify_threshold(const uint16_t* x, int I, uint32_t tau_key, uint16_t* kidx,
+                                      uint16_t* kval, int* count, cudaStream_t st) {
+  const size_t smem = sel_layout(I, 0, 0).end;
+  cudaError_t e = cudaFuncSetAttribute(sparsify_threshold_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  sparsify_threshold_kernel<<<1, SPARSIFY_THREADS, smem, st>>>(x, I, tau_key & 0x7FFFu, kidx, kval, count);
+  return cudaGetLastError();
+}
+
 // ------------------------------------------------------------------------
 // spMspV over the bitmask format (§3 product; §4.1: only the columns of
 // surviving channels are fetched).
@@ -509,8 +533,9 @@ __device__ __forceinline__ Resolved resolve_item(const CmbArgs& a, const ItemCur
   return r;
 }
 
-template <bool FUSED>
+template <int MODE>
 __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArgs a) {
+  constexpr bool FUSED = MODE != CMB_LISTED;   // the kernel builds its own kept list
   extern __shared__ __align__(128) uint8_t sm[];
   __shared__ volatile int abort_flag;
   __shared__ int grid_open;   // 1 once every CTA has zeroed its slice of y
@@ -548,7 +573,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     }
   }
   for (int i = tid; i < 2 * SEG_ROWS; i += CMB_THREADS) tile[i] = 0.f;
-  if (FUSED) select_clear(sel);
+  if (MODE == CMB_TOPK) select_clear(sel);
   // Inputs, y and the grid barrier words may be the previous kernel's.
   griddep_wait();
   if (FUSED) load_x_to_smem(xs, a.x, a.I);
@@ -560,7 +585,19 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   }
   uint32_t u0, u1;   // this CTA's items (32-bit: the launcher keeps counts < 2^31)
   int r0 = 0;        // kept rank of its first item
-  if (a.nruns > 0) {
+  int pr = 0, sr = 0, c0 = 0, c1 = 0;   // threshold mode: run (product, segment), channel range
+  if (MODE == CMB_THRESH) {
+    // Run r (product pr, segment sr) is split into channel ranges; items are
+    // the kept channels of this CTA's range, numbered from 0.
+    int r = 0;
+    while (r + 1 < a.nruns && (unsigned)a.run_cta[r + 1] <= blockIdx.x) ++r;
+    const uint32_t n = a.run_cta[r + 1] - a.run_cta[r], m = blockIdx.x - a.run_cta[r];
+    c0 = (int)((uint32_t)a.I * m / n);
+    c1 = (int)((uint32_t)a.I * (m + 1) / n);
+    sr = r;
+    while (pr < a.np - 1 && sr >= a.p[pr].S) sr -= a.p[pr++].S;
+    u0 = u1 = 0;
+  } else if (a.nruns > 0) {
     int r = 0;
     while (r + 1 < a.nruns && (unsigned)a.run_cta[r + 1] <= blockIdx.x) ++r;
     const uint32_t n = a.run_cta[r + 1] - a.run_cta[r], m = blockIdx.x - a.run_cta[r];
@@ -579,11 +616,24 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       r0 = first.i;
     }
   }
-  const int nv = (int)(u1 - u0);
   // The CTA's items use the kept ranks r0, r0 + 1, ... (mod k): only those
   // entries of the kept list are emitted, at positions 0, 1, ...
   __syncthreads();
-  if (FUSED) select_topk(xs, a.I, a.k, (uint32_t)r0, (uint32_t)a.list_cap, klist, nullptr, sel);
+  if (MODE == CMB_TOPK) select_topk(xs, a.I, a.k, (uint32_t)r0, (uint32_t)a.list_cap, klist, nullptr, sel);
+  if (MODE == CMB_THRESH) u1 = (uint32_t)thresh_compact(xs, c0, c1, a.tau_key, klist, nullptr, sel->wgt);
+  const int nv = (int)(u1 - u0);
+  // An item cursor at item u of this CTA.
+  auto cursor_at = [&](uint32_t u) {
+    ItemCursor c;
+    if (MODE == CMB_THRESH) {
+      c.p = pr;
+      c.s = sr;
+      c.i = (int)u;   // a.k is set above any count, so advance() never wraps
+    } else {
+      c.set(a, u);
+    }
+    return c;
+  };
 
   if (warp == 0) {
     // ---------------- producer ----------------
@@ -591,8 +641,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     const uint64_t pol = policy_evict_first();
     int last_v = -1;
     bool stop = false;
-    ItemCursor cur;
-    cur.set(a, u0 + lane);
+    ItemCursor cur = cursor_at(u0 + lane);
     SlotCursor sc;
     sc.set(lane, nslot);
     Resolved q[PQ];
@@ -707,8 +756,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     uint32_t u = u0;
     int piece = 0;
     while (u < u1) {
-      ItemCursor pc;
-      pc.set(a, u);
+      const ItemCursor pc = cursor_at(u);
       const uint32_t seg_end = u + (uint32_t)(a.k - pc.i);   // end of this (p, s) run
       const uint32_t pend = seg_end < u1 ? seg_end : u1;
       const int va = (int)(u - u0), vb = (int)(pend - u0);
@@ -835,13 +883,15 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   DevProps dp;
   cudaError_t e = dev_props(&dp);
   if (e != cudaSuccess) return e;
-  const bool fused = a.kidx == nullptr;
+  const bool thresh = a.thresh != 0;
+  const bool fused = thresh || a.kidx == nullptr;
   int64_t total = 0;
-  for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * a.k;
+  for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * (thresh ? a.I : a.k);
   if (total <= 0) return cudaSuccess;
   if (total >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;   // item indices are 32-bit
   const int grid = (int)std::min<int64_t>(dp.nsm, total);
   if ((total + grid - 1) / grid >= (int64_t)1 << 30) return cudaErrorInvalidValue;
+  if (thresh) a.k = 1 << 16;   // no rank space: cursors never wrap
   // Item split.  Items are the (problem, segment) runs of k kept channels
   // each, in order.  When every run can have CTAs of its own, runs get CTAs in
   // proportion to their estimated bytes (record = mask + 2 bytes per expected
@@ -875,6 +925,12 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
       per_cta = std::max<int64_t>(per_cta, (a.k + n[q] - 1) / n[q]);
     }
     a.nruns = nruns;
+    if (thresh) {   // channel ranges: at most ceil(I / n) kept per CTA
+      per_cta = 0;
+      for (int q = 0; q < nruns; ++q) per_cta = std::max<int64_t>(per_cta, (a.I + n[q] - 1) / n[q]);
+    }
+  } else if (thresh) {
+    return cudaErrorInvalidValue;   // threshold mode needs CTAs of their own per run
   }
   // Kept-list window of a CTA: at most its item count, at most k.
   a.list_cap = fused ? (int)std::min<int64_t>(per_cta, a.k) : 0;
@@ -894,7 +950,8 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   a.nslot = nslot;
   a.slot_bytes = slot_bytes;
   const size_t smem = cmb_layout(a.I, fused, a.list_cap, nslot, slot_bytes).total;
-  void (*kern)(const CmbArgs) = fused ? cmb_spmspv_kernel<true> : cmb_spmspv_kernel<false>;
+  void (*kern)(const CmbArgs) = thresh ? cmb_spmspv_kernel<CMB_THRESH>
+                                : (fused ? cmb_spmspv_kernel<CMB_TOPK> : cmb_spmspv_kernel<CMB_LISTED>);
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};

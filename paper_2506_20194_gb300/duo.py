@@ -52,6 +52,8 @@ def load_library(path: str | None = None):
     lib.duo_sparsify.argtypes = [vp, i64, i64, vp, vp, vp]
     lib.duo_spmspv.argtypes = [vp, vp, vp, vp, i64, vp, vp]
     lib.duo_spmspv_multi.argtypes = [ctypes.POINTER(vp), i32, vp, vp, vp, i64, ctypes.POINTER(vp), vp]
+    lib.duo_sparsify_threshold.argtypes = [vp, i64, ctypes.c_uint16, vp, vp, vp, vp]
+    lib.duo_spmspv_threshold.argtypes = [ctypes.POINTER(vp), i32, vp, ctypes.c_uint16, ctypes.POINTER(vp), vp]
     lib.duo_free.argtypes = [vp]
     lib.duo_packed_query.argtypes = [vp, ctypes.POINTER(_Info)]
     lib.duo_packed_export.argtypes = [vp, i32, vp, i64]
@@ -61,7 +63,7 @@ def load_library(path: str | None = None):
     lib.duo_strerror.restype = ctypes.c_char_p
     for name in ("duo_pack", "duo_sparsify", "duo_spmspv", "duo_spmspv_multi", "duo_free",
                  "duo_packed_query", "duo_packed_export", "duo_device_status", "duo_abi_version",
-                 "duo_pack_cmb_noalloc"):
+                 "duo_pack_cmb_noalloc", "duo_sparsify_threshold", "duo_spmspv_threshold"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -185,6 +187,42 @@ def duo_spmspv_multi(hs, x: torch.Tensor | None, k: int, kept_idx=None, kept_val
     yarr = (ctypes.c_void_p * n)(*[y.data_ptr() for y in ys])
     _check(load_library().duo_spmspv_multi(harr, n, _ptr(x), _ptr(kept_idx), _ptr(kept_val),
                                            int(k), yarr, _stream_ptr(stream)), "duo_spmspv_multi")
+    return ys
+
+
+def tau_bits(tau) -> int:
+    """fp16 bit pattern of a threshold given as a number or an fp16 tensor."""
+    if isinstance(tau, torch.Tensor):
+        return int(tau.reshape(()).to(torch.float16).view(torch.int16).item()) & 0xFFFF
+    return int(torch.tensor(float(tau), dtype=torch.float16).view(torch.int16).item()) & 0xFFFF
+
+
+def duo_sparsify_threshold(x: torch.Tensor, tau, stream=None):
+    """Channels with |x_j| > |tau| (§5, threshold mask), ascending: returns
+    (kept_idx, kept_val, count) with room for every channel; the first
+    ``count`` (a device int32 tensor) entries are valid."""
+    I = x.numel()
+    kept_idx = torch.empty(I, dtype=torch.int16, device=x.device)
+    kept_val = torch.empty(I, dtype=torch.float16, device=x.device)
+    count = torch.empty(1, dtype=torch.int32, device=x.device)
+    _check(load_library().duo_sparsify_threshold(_ptr(x), I, tau_bits(tau), _ptr(kept_idx),
+                                                 _ptr(kept_val), _ptr(count), _stream_ptr(stream)),
+           "duo_sparsify_threshold")
+    return kept_idx, kept_val, count
+
+
+def duo_spmspv_threshold(hs, x: torch.Tensor, tau, ys=None, stream=None):
+    """y_p = W_p (x ⊙ m^x) with the threshold mask |x_j| > |tau| computed in
+    the launch, for n products sharing x (a list of handles, or one)."""
+    if isinstance(hs, Packed):
+        hs = [hs]
+    n = len(hs)
+    if ys is None:
+        ys = [torch.empty(h.out, dtype=torch.float32, device=x.device) for h in hs]
+    harr = (ctypes.c_void_p * n)(*[h.handle for h in hs])
+    yarr = (ctypes.c_void_p * n)(*[y.data_ptr() for y in ys])
+    _check(load_library().duo_spmspv_threshold(harr, n, _ptr(x), tau_bits(tau), yarr,
+                                               _stream_ptr(stream)), "duo_spmspv_threshold")
     return ys
 
 

@@ -89,6 +89,20 @@ def test_spmspv_rejects_dead_or_fake_handles(lib):
     assert lib.duo_spmspv_multi(arr, 0, FAKE, None, None, 2, arr, None) == EINVAL
 
 
+def test_threshold_entry_points_validate_before_launch(lib):
+    EINVAL = -1
+    arr = (ctypes.c_void_p * 5)(FAKE, FAKE, FAKE, FAKE, FAKE)
+    assert lib.duo_spmspv_threshold(arr, 5, FAKE, 0x3800, arr, None) == EINVAL   # n > 4
+    assert lib.duo_spmspv_threshold(arr, 0, FAKE, 0x3800, arr, None) == EINVAL
+    assert lib.duo_spmspv_threshold(arr, 1, None, 0x3800, arr, None) == EINVAL   # no x
+    assert lib.duo_spmspv_threshold(arr, 1, FAKE, 0x3800, arr, None) == EINVAL   # not a live handle
+    assert lib.duo_sparsify_threshold(None, 16, 0x3800, FAKE, FAKE, FAKE, None) == EINVAL
+    assert lib.duo_sparsify_threshold(FAKE, 0, 0x3800, FAKE, FAKE, FAKE, None) == EINVAL
+    assert lib.duo_sparsify_threshold(FAKE, 65536, 0x3800, FAKE, FAKE, FAKE, None) == EINVAL
+    assert lib.duo_sparsify_threshold(FAKE, 16, 0x3800, FAKE, FAKE, None, None) == EINVAL   # no count
+    assert lib.duo_sparsify_threshold(FAKE + 1, 16, 0x3800, FAKE, FAKE, FAKE, None) == EINVAL   # misaligned
+
+
 def test_free_and_query_reject_non_handles(lib):
     assert lib.duo_free(None) == 0
     assert lib.duo_free(FAKE) == -1
