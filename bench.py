@@ -423,6 +423,8 @@ def run_ours(args):
                               "frac_of_peak": b / (us * 1e-6) / 1e9 / peak, "required_MB": b / 1e6}
             del gs
 
+    thresh = run_threshold_path(duo, shape, layers, args.px, reps, peak)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(shape, layers[0], args.px, args.cpu_seconds)
@@ -445,11 +447,52 @@ def run_ours(args):
             "clocks": clocks,
             "dense_gemv_cublas": dense,
             "sweep_px": sweep,
+            "threshold_path": thresh,
         }
         print(json.dumps(line), flush=True)
     for lay in layers:
         for h in lay["h"].values():
             h.free()
+
+
+def run_threshold_path(duo, shape, layers, px, reps, peak):
+    """The threshold-mask path (§5, threshold-based activation sparsity) on
+    the same layers: per stage a fixed threshold, here the magnitude of the
+    (k+1)-th largest |x| of that layer's input, so that about k channels are
+    kept (all of the top-k set when there is no tie there).  Required bytes
+    use the kept set of the library's own (parity-tested) threshold
+    sparsifier."""
+    L = len(layers)
+    taus, breq = [], 0.0
+    for lay in layers:
+        t = {}
+        for st, src in zip(STAGES, STAGE_SRC):
+            I = shape.I(st[0])
+            k = k_of(I, px)
+            a = lay["x"][src].float().abs()
+            t[src] = float(torch.sort(a, descending=True).values[k].item()) if k < I else -1.0
+            tau = max(t[src], 0.0)
+            idx, _, cnt = duo.duo_sparsify_threshold(lay["x"][src], tau)
+            n = int(cnt.item())
+            K = idx[:n].to(torch.int64) & 0xFFFF
+            for p in st:
+                breq += float(lay["nnz"][p][K].sum().item()) * 2.0 + n * shape.O(p) / 8.0 + 4.0 * shape.O(p)
+            breq += 2.0 * I + 4.0 * n
+        taus.append(t)
+    breq /= L
+
+    def fn():
+        for lay, t in zip(layers, taus):
+            for st, src in zip(STAGES, STAGE_SRC):
+                duo.duo_spmspv_threshold([lay["h"][p] for p in st], lay["x"][src], max(t[src], 0.0),
+                                         ys=[lay["y"][p] for p in st])
+    g = capture(fn)
+    time_graph(g, 3)
+    r = max(3, min(reps, 500))
+    us = time_graph(g, r) / (r * L) * 1e6
+    gbs = breq / (us * 1e-6) / 1e9
+    return {"us_per_layer": us, "GB/s": gbs, "frac_of_peak": gbs / peak, "required_MB": breq / 1e6,
+            "tau": "magnitude of the (k+1)-th largest |x| of each stage input, fixed before timing"}
 
 
 def run_e2e(duo, shape, layers, args, breq_mean):

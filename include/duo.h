@@ -8,7 +8,7 @@
  *
  * where W (O rows x I input channels, fp16) carries unstructured weight
  * sparsity (pruned entries are stored as zero, §3 mask m^w) and m^x keeps the
- * k input channels of largest |x_i|, chosen "on the fly" (§3).  §4.1
+ * k input channels of largest |x_i|, chosen per input at decode time (§3).  §4.1
  * describes the execution: only the compressed weight columns of the
  * surviving channels are fetched from HBM.
  *

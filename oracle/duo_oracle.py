@@ -6,7 +6,7 @@ Notation follows the paper (DuoGPT, arXiv 2506.20194, §3 "Preliminaries"):
 the layer weight is W in R^{n x k} with n output rows and k input channels
 (here O = n rows, I = k channels, to keep the letter k for the number of kept
 channels), the input is a column vector x, and activation sparsity multiplies
-x by a binary mask m^x chosen by magnitude "on the fly" (§3, "Activation
+x by a binary mask m^x chosen by magnitude at decode time (§3, "Activation
 Sparsity").  The decode-time product is
 
     y = W (x ⊙ m^x) = sum_{i : m^x_i = 1} W[:, i] * x_i          (§3)
