@@ -31,6 +31,7 @@ struct duo_packed {
   void* data;
   int64_t data_bytes;
   unsigned int* sync;  // BITMASK: 2-word grid barrier of the spMspV kernel
+  uint16_t* kept;      // BITMASK: room for a kept list (ids, then values; 2 x in each)
   int max_record;      // BITMASK: bytes of the largest record
 };
 
@@ -186,9 +187,12 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
     // The offsets are followed (at a 256-byte boundary) by the two barrier
     // words of the spMspV kernel, zeroed here.
     const size_t sync_at = (size_t)(h->index_bytes + 255) / 256 * 256;
-    e = duo_malloc(&index, sync_at + 256);
+    // after the offsets: the grid barrier words, then a kept-list buffer for
+    // launches with more (product, segment) runs than SMs (selection first)
+    e = duo_malloc(&index, sync_at + 256 + (size_t)(4 * in + 15) / 16 * 16);
     if (e != cudaSuccess) return fail(map_err(e));
     h->sync = reinterpret_cast<unsigned int*>(static_cast<char*>(index) + sync_at);
+    h->kept = reinterpret_cast<uint16_t*>(static_cast<char*>(index) + sync_at + 256);
     e = cudaMemsetAsync(h->sync, 0, 256, st);
     if (e != cudaSuccess) return fail(map_err(e));
     e = duo::launch_cmb_offsets(cnt_js, in * S, static_cast<uint32_t*>(index), totals, st);
@@ -371,6 +375,17 @@ static int spmspv_common(const duo_packed* const* hs, int n, const void* x, cons
       a.p[p].dens = (float)((double)hs[p]->nnz / ((double)hs[p]->out * (double)hs[p]->in));
     }
     e = duo::launch_cmb_spmspv(a, st);
+    if (e == cudaErrorNotSupported) {
+      // More (product, segment) runs than SMs: select into the first
+      // handle's kept-list buffer, then launch with that list.
+      uint16_t* kidx2 = hs[0]->kept;
+      uint16_t* kval2 = hs[0]->kept + I;
+      e = duo::launch_sparsify(static_cast<const uint16_t*>(x), (int)I, (int)k, kidx2, kval2, st);
+      if (e != cudaSuccess) return map_err(e);
+      a.kidx = kidx2;
+      a.kval = kval2;
+      e = duo::launch_cmb_spmspv(a, st);
+    }
     if (e == cudaErrorInvalidValue) return DUO_ERANGE;
   } else {
     const duo_packed* h = hs[0];

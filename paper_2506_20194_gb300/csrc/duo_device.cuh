@@ -277,80 +277,52 @@ constexpr int SEL_MAX_WARPS = 32;
 // Shared state of the selection.
 struct SelShared {
   uint32_t hist[SEL_BINS];
-  uint32_t subw[SEL_MAX_WARPS][16];   // per warp: its keys of bin C by key & 15
-  uint32_t wgt[SEL_MAX_WARPS];        // per warp: its keys in bins above C
-  uint32_t wpre[SEL_MAX_WARPS];       // per warp: keys above T | ties << 16 in lower warps
-  uint32_t wown[SEL_MAX_WARPS];       // per warp: its own keys above T | ties << 16
-  uint32_t C, aboveC, T, q;
+  uint32_t sub[16];               // keys of bin C by key & 15
+  uint32_t wcnt[SEL_MAX_WARPS];   // per-warp counts
+  uint32_t C, aboveC;
+  int T, cut;                     // the selection's result (see select_threshold)
 };
 
-// Clears the histograms (before the __syncthreads that precedes select_topk).
+// Clears the histograms (before the __syncthreads that precedes the selection).
 __device__ __forceinline__ void select_clear(SelShared* sh) {
   uint4* h = reinterpret_cast<uint4*>(sh->hist);
-  for (int i = threadIdx.x; i < (SEL_BINS + 16 * SEL_MAX_WARPS) / 4; i += blockDim.x)
-    h[i] = make_uint4(0u, 0u, 0u, 0u);   // hist and subw are contiguous
+  for (int i = threadIdx.x; i < (SEL_BINS + 16) / 4; i += blockDim.x)
+    h[i] = make_uint4(0u, 0u, 0u, 0u);   // hist and sub are contiguous
 }
 
-// Exact top-k by magnitude (§3): keeps the k channels with the largest
-// |x_j|, ties to the lower index.  The key of x_j is its fp16 bit pattern
-// with the sign cleared; for IEEE fp16 this integer order equals the order of
-// |x_j| (NaN patterns sort above Inf).  xs holds the fp16 bits of x in
-// shared memory (room for a whole number of 32-channel words).
+// The key of x_j is its fp16 bit pattern with the sign cleared; for IEEE
+// fp16 this integer order equals the order of |x_j| (NaN patterns sort above
+// Inf).
+__device__ __forceinline__ int key_of(const uint16_t* xs, int j) { return xs[j] & 0x7FFF; }
+
+// Exact top-k by magnitude (§3) as a threshold: keeps the k channels with
+// the largest |x_j|, ties to the lower index.  On return (to every thread)
+// channel j is kept iff key_j > T, or key_j == T and j <= cut.
 //
 //  1. histogram of key >> 4 (2048 bins, shared-memory atomics);
-//  2. one warp finds, by suffix scans over 32 blocks of 64 bins and then
-//     over the bins of the block that holds the crossing, the bin C where the
-//     count from the top reaches k;
-//  3. warp w walks its contiguous run of 32-channel words (lane = channel)
-//     and counts its keys in bins above C (ballots) and, by key & 15, its
-//     keys in bin C (its own 16 counters);
-//  4. one warp sums the per-warp counters of bin C to find the threshold
-//     key T = 16 C + b and q = k - count(key > T), the number of channels
-//     with key == T that are kept (the lowest-indexed ones), and scans the
-//     per-warp counts to give every warp the "above T" and "tie" counts
-//     before its own run;
-//  5. warps whose kept ranks meet the requested window walk their words
-//     again: kept channel j has rank r = (channels above T before j) +
-//     min(q, ties before j); if d = (r - r0) mod k is below rn it writes
-//     klist[d] = j and kvals[d] = its fp16 bits.
-//
-// The window is the cyclic rank range r0, r0 + 1, ... (mod k) of length
-// min(rn, k); with r0 = 0 and rn = k the lists are indexed by rank.
-//
-// select_clear() and the loading of xs come first, then a __syncthreads.
-// All threads of the block take part (512 <= blockDim.x <= 1024, a multiple
-// of 32); it ends with a __syncthreads.
-constexpr uint32_t KEY_NONE = 0xFFFFu;
-__device__ __forceinline__ uint32_t key_of(const uint16_t* xs, int j) { return xs[j] & 0x7FFFu; }
-
-__device__ __forceinline__ bool ranges_meet(uint32_t a0, uint32_t a1, uint32_t b0, uint32_t b1) {
-  return a0 < b1 && b0 < a1;
-}
-
-__device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t r0, uint32_t rn,
-                                   uint16_t* klist, uint16_t* kvals, SelShared* sh) {
+//  2. one warp finds the bin C where the count from the top reaches k: a
+//     suffix scan over 32 lanes x 64 bins, then over the 64 bins of the
+//     crossing lane (2 per lane);
+//  3. histogram of key & 15 over the keys of bin C (few: contention-free
+//     atomics);
+//  4. one warp gets T = 16 C + b and q = k - count(key > T), the number of
+//     channels with key == T to keep (the lowest-indexed ones);
+//  5. only if fewer than all of them are kept: each warp counts the ties in
+//     its contiguous run of 32-channel words, and the warp holding the q-th
+//     tie finds its channel, cut; otherwise cut = I.
+// k <= 0 keeps nothing (T = 0x7FFF, cut = -1), k >= I everything (T = -1).
+// xs holds the fp16 bits of x (room for a whole number of 32-channel words);
+// select_clear() and the loading of xs come first, then a __syncthreads.  All
+// threads of the block take part (512 <= blockDim.x <= 1024, a multiple of
+// 32); it ends with a __syncthreads.
+__device__ inline void select_threshold(const uint16_t* xs, int I, int k, SelShared* sh, int* T_out,
+                                        int* cut_out) {
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, wid = tid >> 5;
   const int nwarps = nt >> 5;
-  const int nw = (I + 31) >> 5;
   const uint32_t kk = (uint32_t)k;
-  const bool whole = rn >= kk;
-  // list position of rank r, or -1 outside the window
-  auto slot_of = [&](uint32_t r) -> int {
-    const uint32_t d = r >= r0 ? r - r0 : r + kk - r0;
-    return (whole || d < rn) ? (int)d : -1;
-  };
-  if (k <= 0) {   // nothing kept
-    __syncthreads();
-    return;
-  }
-  if (k >= I) {   // everything kept: rank = channel
-    for (int j = tid; j < I; j += nt) {
-      const int d = slot_of((uint32_t)j);
-      if (d >= 0) {
-        if (klist != nullptr) klist[d] = (uint16_t)j;
-        if (kvals != nullptr) kvals[d] = xs[j];
-      }
-    }
+  if (k <= 0 || k >= I) {
+    *T_out = k <= 0 ? 0x7FFF : -1;   // no key exceeds 0x7FFF; every key exceeds -1
+    *cut_out = -1;
     __syncthreads();
     return;
   }
@@ -358,8 +330,8 @@ __device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t r0
   {
     int j = tid;
     for (; j + 3 * nt < I; j += 4 * nt) {
-      const uint32_t k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
-      const uint32_t k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
+      const int k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
+      const int k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
       atomicAdd(&sh->hist[k0 >> 4], 1u);
       atomicAdd(&sh->hist[k1 >> 4], 1u);
       atomicAdd(&sh->hist[k2 >> 4], 1u);
@@ -368,9 +340,7 @@ __device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t r0
     for (; j < I; j += nt) atomicAdd(&sh->hist[key_of(xs, j) >> 4], 1u);
   }
   __syncthreads();
-  // 2. threshold bin C, by warp 0 alone: lane l totals bins [64 l, 64 l + 64),
-  //    a suffix scan over lanes finds the lane whose bins hold the crossing,
-  //    and a second scan over that lane's 64 bins (2 per lane) finds C.
+  // 2. threshold bin C, by warp 0
   if (wid == 0) {
     const uint4* h4 = reinterpret_cast<const uint4*>(sh->hist) + 16 * lane;
     uint32_t s64 = 0;
@@ -404,40 +374,29 @@ __device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t r0
     }
   }
   __syncthreads();
-  // 3. per-warp counts over the warp's words [w0, w1)
-  const int per = (nw + nwarps - 1) / nwarps;
-  const int w0 = min(nw, wid * per), w1 = min(nw, w0 + per);
+  // 3. the 16 keys of bin C
   {
-    const uint32_t C = sh->C;
-    uint32_t ngt = 0;
-    for (int w = w0; w < w1; w += 4) {
-      uint32_t key[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int j = 32 * (w + u) + lane;
-        key[u] = (w + u < w1 && j < I) ? key_of(xs, j) : KEY_NONE;
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const bool valid = key[u] != KEY_NONE;
-        ngt += (uint32_t)__popc(__ballot_sync(FULL_MASK, valid && (key[u] >> 4) > C));
-        if (valid && (key[u] >> 4) == C) atomicAdd(&sh->subw[wid][key[u] & 15u], 1u);
-      }
+    const int C = (int)sh->C;
+    int j = tid;
+    for (; j + 3 * nt < I; j += 4 * nt) {
+      const int k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
+      const int k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
+      if ((k0 >> 4) == C) atomicAdd(&sh->sub[k0 & 15], 1u);
+      if ((k1 >> 4) == C) atomicAdd(&sh->sub[k1 & 15], 1u);
+      if ((k2 >> 4) == C) atomicAdd(&sh->sub[k2 & 15], 1u);
+      if ((k3 >> 4) == C) atomicAdd(&sh->sub[k3 & 15], 1u);
     }
-    if (lane == 0) sh->wgt[wid] = ngt;
+    for (; j < I; j += nt) {
+      const int key = key_of(xs, j);
+      if ((key >> 4) == C) atomicAdd(&sh->sub[key & 15], 1u);
+    }
   }
   __syncthreads();
-  // 4. by warp 0 alone: the threshold key T = 16 C + b (lane v < 16 = key & 15
-  //    inside bin C), q, and for every warp w (lane w) its own and its lower
-  //    warps' counts above T and equal to T.
-  if (wid == 0) {
-    uint32_t part[4] = {0u, 0u, 0u, 0u};
-    if (lane < 16) {
-#pragma unroll
-      for (int w = 0; w < SEL_MAX_WARPS; ++w)
-        if (w < nwarps) part[w & 3] += sh->subw[w][lane];
-    }
-    const uint32_t sv = (part[0] + part[1]) + (part[2] + part[3]);
+  // 4. T and q (lane v < 16 = key & 15 inside bin C), by every warp: the
+  //    result is read by all, with no further barrier.
+  int T, q, ties;
+  {
+    const uint32_t sv = lane < 16 ? sh->sub[lane] : 0u;
     uint32_t suf = sv;   // keys of bin C with key & 15 >= lane
 #pragma unroll
     for (int o = 1; o < 16; o <<= 1) {
@@ -446,102 +405,65 @@ __device__ inline void select_topk(const uint16_t* xs, int I, int k, uint32_t r0
     }
     const uint32_t need = kk - sh->aboveC;   // >= 1, <= hist[C]
     const int b = 31 - __clz(__ballot_sync(FULL_MASK, lane < 16 && suf >= need));
-    const uint32_t above_in_c = __shfl_sync(FULL_MASK, suf - sv, b);
-    uint32_t al = 0, tl = 0;
-    if (lane < nwarps) {
-      const uint4* row = reinterpret_cast<const uint4*>(sh->subw[lane]);
-      al = sh->wgt[lane];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int c = (i + (lane >> 1)) & 3;   // rotated: conflict-free quarter warps
-        const uint4 r4 = row[c];
-        const uint32_t v4[4] = {r4.x, r4.y, r4.z, r4.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int v = 4 * c + e;
-          al += v > b ? v4[e] : 0u;
-          tl += v == b ? v4[e] : 0u;
+    T = 16 * (int)sh->C + b;
+    q = (int)(need - __shfl_sync(FULL_MASK, suf - sv, b));   // >= 1
+    ties = (int)__shfl_sync(FULL_MASK, sv, b);
+  }
+  int cut = I;
+  if (q < ties) {
+    // 5. the q-th channel with key == T in index order
+    const int nw = (I + 31) >> 5;
+    const int per = (nw + nwarps - 1) / nwarps;
+    const int w0 = min(nw, wid * per), w1 = min(nw, w0 + per);
+    uint32_t cnt = 0;
+    for (int w = w0; w < w1; ++w) {
+      const int j = 32 * w + lane;
+      cnt += (uint32_t)__popc(__ballot_sync(FULL_MASK, j < I && key_of(xs, j) == T));
+    }
+    if (lane == 0) sh->wcnt[wid] = cnt;
+    __syncthreads();
+    const uint32_t c = lane < nwarps ? sh->wcnt[lane] : 0u;   // lane l: warp l's count
+    uint32_t before = __reduce_add_sync(FULL_MASK, lane < wid ? c : 0u);
+    const uint32_t own = __shfl_sync(FULL_MASK, c, wid);   // this warp's count, in every lane
+    if (before < (uint32_t)q && (uint32_t)q <= before + own) {   // this warp holds the q-th tie
+      for (int w = w0; w < w1; ++w) {
+        const int j = 32 * w + lane;
+        const uint32_t m = __ballot_sync(FULL_MASK, j < I && key_of(xs, j) == T);
+        const uint32_t n = (uint32_t)__popc(m);
+        if (before + n >= (uint32_t)q) {
+          if (lane == 0) sh->cut = 32 * w + select_bit(m, q - 1 - (int)before);
+          break;
         }
+        before += n;
       }
     }
-    const uint32_t own = al | (tl << 16);   // each <= 65535
-    const uint32_t pre = warp_inclusive_scan(own, lane) - own;
-    if (lane < nwarps) {
-      sh->wpre[lane] = pre;
-      sh->wown[lane] = own;
-    }
-    if (lane == 0) {
-      sh->T = 16u * sh->C + (uint32_t)b;
-      sh->q = need - above_in_c;   // >= 1
-    }
+    __syncthreads();
+    cut = sh->cut;
   }
-  __syncthreads();
-  const uint32_t T = sh->T, q = sh->q;
-  uint32_t gpre, epre, a_own, t_own;
-  {
-    const uint32_t pre = sh->wpre[wid], own = sh->wown[wid];
-    gpre = pre & 0xFFFFu;
-    epre = pre >> 16;
-    a_own = own & 0xFFFFu;
-    t_own = own >> 16;
-  }
-  // 5. emission by the warps whose kept ranks meet the window
-  if (klist != nullptr || kvals != nullptr) {
-    const uint32_t R = gpre + min(epre, q);
-    const uint32_t Kw = a_own + min(epre + t_own, q) - min(epre, q);
-    bool meet = whole;
-    if (!meet && Kw > 0) {
-      const uint32_t e0 = r0 + rn;   // window [r0, e0), wrapping past kk
-      meet = ranges_meet(R, R + Kw, r0, min(e0, kk)) || (e0 > kk && ranges_meet(R, R + Kw, 0u, e0 - kk));
-    }
-    if (meet) {
-      const uint32_t lt = (1u << lane) - 1u;
-      for (int w = w0; w < w1; w += 4) {
-        uint32_t key[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int j = 32 * (w + u) + lane;
-          key[u] = (w + u < w1 && j < I) ? key_of(xs, j) : KEY_NONE;
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const bool valid = key[u] != KEY_NONE;
-          const bool isg = valid && key[u] > T;
-          const bool ise = valid && key[u] == T;
-          const uint32_t g = __ballot_sync(FULL_MASK, isg);
-          const uint32_t e = __ballot_sync(FULL_MASK, ise);
-          const uint32_t tr = epre + (uint32_t)__popc(e & lt);   // ties before this channel
-          if (isg || (ise && tr < q)) {
-            const int d = slot_of(gpre + (uint32_t)__popc(g & lt) + min(tr, q));
-            if (d >= 0) {
-              const int j = 32 * (w + u) + lane;
-              if (klist != nullptr) klist[d] = (uint16_t)j;
-              if (kvals != nullptr) kvals[d] = xs[j];
-            }
-          }
-          gpre += (uint32_t)__popc(g);
-          epre += (uint32_t)__popc(e);
-        }
-      }
-    }
-  }
+  *T_out = T;
+  *cut_out = cut;
   __syncthreads();
 }
 
-// Threshold mask (§5, threshold-based activation sparsity): writes the
-// channels j in [c0, c1) with key_j > T in ascending order to klist[0..n) (and
-// their fp16 bits to kvals if given) and returns n to every thread.  Warps
-// take contiguous runs of the range's 32-channel words (lane = channel): one
+// Writes the channels j in [c0, c1) that a threshold keeps (key_j > T, or
+// key_j == T and j <= cut) in ascending order to klist[0..n) (and their fp16
+// bits to kvals if given) and returns n to every thread.  Warps take
+// contiguous runs of the range's 32-channel words (lane = channel): one
 // ballot pass counts, a block barrier and a sum over lower warps place each
 // warp's run, a second pass writes.  wcnt needs one entry per warp.  All
-// threads take part; it ends with a __syncthreads.
-__device__ inline int thresh_compact(const uint16_t* xs, int c0, int c1, uint32_t T, uint16_t* klist,
-                                     uint16_t* kvals, uint32_t* wcnt) {
+// threads take part; it ends with a __syncthreads.  Used for the threshold
+// mask of §5 (T = tau, cut = -1) and for the top-k set as a threshold.
+__device__ inline int thresh_compact(const uint16_t* xs, int c0, int c1, int T, int cut,
+                                     uint16_t* klist, uint16_t* kvals, uint32_t* wcnt) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   const int wb = c0 >> 5, nwd = c1 > c0 ? ((c1 + 31) >> 5) - wb : 0;
   const int per = (nwd + nwarps - 1) / nwarps;
   const int w0 = wb + min(nwd, wid * per), w1 = wb + min(nwd, wid * per + per);
-  auto kept = [&](int j) { return j >= c0 && j < c1 && key_of(xs, j) > T; };
+  auto kept = [&](int j) {
+    if (j < c0 || j >= c1) return false;
+    const int key = key_of(xs, j);
+    return key > T || (key == T && j <= cut);
+  };
   uint32_t cnt = 0;
   for (int w = w0; w < w1; ++w) cnt += (uint32_t)__popc(__ballot_sync(FULL_MASK, kept(32 * w + lane)));
   if (lane == 0) wcnt[wid] = cnt;

@@ -318,7 +318,9 @@ __global__ void __launch_bounds__(SPARSIFY_THREADS) sparsify_kernel(const uint16
   load_x_to_smem(xs, x, I);
   select_clear(sel);
   __syncthreads();
-  select_topk(xs, I, k, 0u, (uint32_t)k, kidx, kval, sel);
+  int T, cut;
+  select_threshold(xs, I, k, sel, &T, &cut);
+  thresh_compact(xs, 0, I, T, cut, kidx, kval, sel->wcnt);
 }
 
 cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uint16_t* kval,
@@ -341,7 +343,7 @@ __global__ void __launch_bounds__(SPARSIFY_THREADS) sparsify_threshold_kernel(
   SelShared* sel = reinterpret_cast<SelShared*>(sm + L.sel);
   load_x_to_smem(xs, x, I);
   __syncthreads();
-  const int n = thresh_compact(xs, 0, I, T, kidx, kval, sel->wgt);
+  const int n = thresh_compact(xs, 0, I, (int)T, -1, kidx, kval, sel->wcnt);
   if (threadIdx.x == 0) *count = n;
 }
 
@@ -585,8 +587,8 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   }
   uint32_t u0, u1;   // this CTA's items (32-bit: the launcher keeps counts < 2^31)
   int r0 = 0;        // kept rank of its first item
-  int pr = 0, sr = 0, c0 = 0, c1 = 0;   // threshold mode: run (product, segment), channel range
-  if (MODE == CMB_THRESH) {
+  int pr = 0, sr = 0, c0 = 0, c1 = 0;   // fused modes: run (product, segment), channel range
+  if (FUSED) {
     // Run r (product pr, segment sr) is split into channel ranges; items are
     // the kept channels of this CTA's range, numbered from 0.
     int r = 0;
@@ -610,25 +612,23 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     for (int p = 0; p < a.np; ++p) total += (uint32_t)a.p[p].S * (uint32_t)a.k;
     u0 = (uint32_t)((uint64_t)total * blockIdx.x / gridDim.x);
     u1 = (uint32_t)((uint64_t)total * (blockIdx.x + 1) / gridDim.x);
-    if (FUSED) {
-      ItemCursor first;
-      first.set(a, u0);
-      r0 = first.i;
-    }
   }
-  // The CTA's items use the kept ranks r0, r0 + 1, ... (mod k): only those
-  // entries of the kept list are emitted, at positions 0, 1, ...
   __syncthreads();
-  if (MODE == CMB_TOPK) select_topk(xs, a.I, a.k, (uint32_t)r0, (uint32_t)a.list_cap, klist, nullptr, sel);
-  if (MODE == CMB_THRESH) u1 = (uint32_t)thresh_compact(xs, c0, c1, a.tau_key, klist, nullptr, sel->wgt);
+  if (FUSED) {
+    // The kept set as a threshold (top-k: computed here; threshold mask:
+    // given), then this CTA's kept channels of its range, numbered from 0.
+    int T = (int)a.tau_key, cut = -1;
+    if (MODE == CMB_TOPK) select_threshold(xs, a.I, a.k, sel, &T, &cut);
+    u1 = (uint32_t)thresh_compact(xs, c0, c1, T, cut, klist, nullptr, sel->wcnt);
+  }
   const int nv = (int)(u1 - u0);
   // An item cursor at item u of this CTA.
   auto cursor_at = [&](uint32_t u) {
     ItemCursor c;
-    if (MODE == CMB_THRESH) {
+    if (FUSED) {
       c.p = pr;
       c.s = sr;
-      c.i = (int)u;   // a.k is set above any count, so advance() never wraps
+      c.i = (int)u;   // u < nv <= k (top-k) or a.k above any count: advance() never wraps
     } else {
       c.set(a, u);
     }
@@ -892,12 +892,15 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   const int grid = (int)std::min<int64_t>(dp.nsm, total);
   if ((total + grid - 1) / grid >= (int64_t)1 << 30) return cudaErrorInvalidValue;
   if (thresh) a.k = 1 << 16;   // no rank space: cursors never wrap
-  // Item split.  Items are the (problem, segment) runs of k kept channels
-  // each, in order.  When every run can have CTAs of its own, runs get CTAs in
+  // Item split.  Items are the (problem, segment) runs of kept channels, in
+  // order.  When every run can have CTAs of its own, runs get CTAs in
   // proportion to their estimated bytes (record = mask + 2 bytes per expected
   // non-zero) and no CTA spans two runs: a run boundary inside a CTA would
-  // cost a mid-stream flush of all its consumers' rows.  Otherwise the items
-  // are split evenly.
+  // cost a mid-stream flush of all its consumers' rows.  A CTA of a fused mode
+  // takes a channel range of its run (the kept set is a threshold, so it can
+  // find its own kept channels); with a kept list it takes a rank range.
+  // Otherwise (more runs than CTAs) a kept list is split evenly, and the
+  // fused modes are not launched.
   int nruns = 0;
   for (int p = 0; p < a.np; ++p) nruns += a.p[p].S;
   int64_t per_cta = (total + grid - 1) / grid;
@@ -925,12 +928,14 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
       per_cta = std::max<int64_t>(per_cta, (a.k + n[q] - 1) / n[q]);
     }
     a.nruns = nruns;
-    if (thresh) {   // channel ranges: at most ceil(I / n) kept per CTA
+    if (fused) {   // channel ranges: at most ceil(I / n) kept per CTA
       per_cta = 0;
       for (int q = 0; q < nruns; ++q) per_cta = std::max<int64_t>(per_cta, (a.I + n[q] - 1) / n[q]);
     }
   } else if (thresh) {
-    return cudaErrorInvalidValue;   // threshold mode needs CTAs of their own per run
+    return cudaErrorInvalidValue;   // the fused modes need CTAs of their own per run
+  } else if (fused) {
+    return cudaErrorNotSupported;   // the caller selects first and launches with a kept list
   }
   // Kept-list window of a CTA: at most its item count, at most k.
   a.list_cap = fused ? (int)std::min<int64_t>(per_cta, a.k) : 0;
@@ -993,7 +998,9 @@ __global__ void __launch_bounds__(IDX16_THREADS, 1) idx16_spmspv_kernel(const Id
     load_x_to_smem(xs, a.x, a.I);
     select_clear(sel);
     __syncthreads();
-    select_topk(xs, a.I, a.k, 0u, (uint32_t)a.k, klist, nullptr, sel);
+    int T, cut;
+    select_threshold(xs, a.I, a.k, sel, &T, &cut);
+    thresh_compact(xs, 0, a.I, T, cut, klist, nullptr, sel->wcnt);
   }
   const int nwt = gridDim.x * (IDX16_THREADS / 32);
   for (int i = blockIdx.x * (IDX16_THREADS / 32) + warp; i < a.k; i += nwt) {
