@@ -36,8 +36,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch of
 # the fused kernel from one ncu capture, valid only for the kernel source it
 # was taken on (sha256 of kernels.cu + duo_device.cuh, first 16 hex digits).
-TRAFFIC = {"sha": "485b3751699d2b20",
-           "per_launch_bytes": [29127680.0, 9773312.0, 51913984.0, 26120960.0]}
+TRAFFIC = {"sha": "05dc308352cf79df",
+           "per_launch_bytes": [29106176.0, 9754624.0, 51912448.0, 26100736.0]}
 
 
 def parse():
