@@ -31,4 +31,15 @@ from .duo_oracle import (  # noqa: F401
     required_bytes,
     loaded_fraction,
     worst_case_loaded_fraction,
+    QUANT_GROUP,
+    QUANT_BITS,
+    oracle_quantize_rtn,
+    oracle_dequantize,
+    oracle_spmspv_q,
+    oracle_spmspv_q_threshold,
+    exact_spmspv_q_rows_scaled,
+    tolerance_rows_f64,
+    ref_pack_cmb_q,
+    ref_unpack_cmb_q,
+    required_bytes_q,
 )

@@ -333,3 +333,237 @@ def worst_case_loaded_fraction(nnz_per_channel, k: int, O: int, I: int) -> float
     """Upper bound of App. B.3: the k densest channels are the ones kept."""
     n = np.sort(np.asarray(nnz_per_channel, dtype=np.float64))[::-1]
     return float(n[:k].sum() / (O * I))
+
+
+# --------------------------------------------------------------------------
+# Weight-only quantisation of the stored values (§5, compatibility with
+# weight-only quantisation, Table 4): b-bit uniform integers (b = 8 or 4),
+# round-to-nearest ("RTN", no error feedback), one grid per output row and
+# group of 128 consecutive input channels.
+#
+# Readings (the paper names only "uniform integer", "channel-wise RTN" and the
+# group size; it follows the GPTQ / OBC line of work, whose quantiser is the
+# asymmetric min-max grid):
+#   * per (row i, group g): lo = min(0, min W), hi = max(0, max W) over the
+#     group's entries; scale s = (hi - lo) / (2**b - 1), computed in fp64 and
+#     rounded to the nearest fp16 (ties to even); s = 1 for a group with no
+#     non-zero entry, s = 2**-24 if a non-zero quotient rounds to 0;
+#   * zero point z = rint(-lo / s) (ties to even), clamped to [0, 2**b - 1];
+#   * code q = clamp(rint(w / s) + z, 0, 2**b - 1) for every stored (non-zero)
+#     entry, the quotients in fp64; pruned entries stay pruned (no code, mask
+#     bit 0), and a code equal to z keeps its mask bit although it stands for 0;
+#   * the dequantised weight is s * (q - z) (exact in fp64); y sums it against
+#     x over the kept channels in fp64.
+# --------------------------------------------------------------------------
+
+QUANT_GROUP = 128
+QUANT_BITS = (8, 4)
+
+
+def _check_bits(bits):
+    if bits not in QUANT_BITS:
+        raise ValueError(f"bits must be one of {QUANT_BITS}")
+    return (1 << bits) - 1
+
+
+def oracle_quantize_rtn(W16, bits: int):
+    """RTN quantisation of the non-zero entries of W (readings above).
+
+    Returns ``(q, s16, z)``: q int64 O x I (the code of every non-zero entry,
+    0 where pruned), s16 float16 O x G and z int64 O x G with
+    G = ceil(I / 128); group g holds channels 128 g .. 128 g + 127.
+    """
+    W = _as_f16(W16)
+    if W.ndim != 2:
+        raise ValueError("W must be O x I")
+    maxq = _check_bits(bits)
+    O, I = W.shape
+    G = (I + QUANT_GROUP - 1) // QUANT_GROUP
+    nz = (W.view(np.uint16) & 0x7FFF) != 0
+    Wd = np.where(nz, W.astype(np.float64), 0.0)
+    q = np.zeros((O, I), dtype=np.int64)
+    s16 = np.zeros((O, G), dtype=np.float16)
+    z = np.zeros((O, G), dtype=np.int64)
+    for g in range(G):
+        c0, c1 = g * QUANT_GROUP, min(I, (g + 1) * QUANT_GROUP)
+        blk = Wd[:, c0:c1]
+        lo = np.minimum(blk.min(axis=1), 0.0)
+        hi = np.maximum(blk.max(axis=1), 0.0)
+        sg = ((hi - lo) / maxq).astype(np.float16)
+        empty = hi == lo
+        sg[empty] = np.float16(1.0)
+        sg[(sg == 0) & ~empty] = np.uint16(1).view(np.float16)   # 2**-24
+        sd = sg.astype(np.float64)
+        zg = np.clip(np.rint(-lo / sd), 0, maxq).astype(np.int64)
+        qg = np.clip(np.rint(blk / sd[:, None]) + zg[:, None], 0, maxq).astype(np.int64)
+        q[:, c0:c1] = np.where(nz[:, c0:c1], qg, 0)
+        s16[:, g] = sg
+        z[:, g] = zg
+    return q, s16, z
+
+
+def oracle_dequantize(W16, bits: int) -> np.ndarray:
+    """The weight the quantised store stands for: s * (q - z) at every
+    non-zero entry of W, 0 at pruned ones (fp64, exact)."""
+    W = _as_f16(W16)
+    q, s16, z = oracle_quantize_rtn(W, bits)
+    g = np.arange(W.shape[1]) // QUANT_GROUP
+    nz = (W.view(np.uint16) & 0x7FFF) != 0
+    deq = s16.astype(np.float64)[:, g] * (q - z[:, g]).astype(np.float64)
+    return np.where(nz, deq, 0.0)
+
+
+def oracle_spmspv_q(W16, x16, k: int, bits: int) -> np.ndarray:
+    """y = W_q (x ⊙ m^x) in fp64 with the top-k mask (§3) and the RTN-quantised
+    weight of :func:`oracle_dequantize` (§5, Table 4)."""
+    Wq = oracle_dequantize(W16, bits)
+    K, xv = oracle_sparsify(x16, k)
+    if Wq.shape[1] != _as_f16(x16).size:
+        raise ValueError("W and x disagree on I")
+    return Wq[:, K.astype(np.int64)] @ xv.astype(np.float64)
+
+
+def oracle_spmspv_q_threshold(W16, x16, tau, bits: int) -> np.ndarray:
+    """As :func:`oracle_spmspv_q` with the threshold mask of
+    :func:`oracle_sparsify_threshold`."""
+    Wq = oracle_dequantize(W16, bits)
+    K, xv = oracle_sparsify_threshold(x16, tau)
+    if Wq.shape[1] != _as_f16(x16).size:
+        raise ValueError("W and x disagree on I")
+    return Wq[:, K.astype(np.int64)] @ xv.astype(np.float64)
+
+
+def exact_spmspv_q_rows_scaled(q_rows, s16_rows, z_rows, nz_rows, x16, K) -> list[int]:
+    """Exact y_i * 2**48 as Python integers from the codes themselves: every
+    fp16 scale is an integer multiple of 2**-24, so
+    y_i * 2**48 = sum_j (s_ig * 2**24) * (q_ij - z_ig) * (x_j * 2**24)."""
+    x = _as_f16(x16).reshape(-1)
+    s_int = (np.asarray(s16_rows, dtype=np.float16).astype(np.float64) * 2.0**24).astype(np.int64)
+    out = []
+    for r in range(len(q_rows)):
+        acc = 0
+        for j in (int(c) for c in K):
+            if not nz_rows[r][j]:
+                continue
+            g = j // QUANT_GROUP
+            xi = int(float(x[j]) * 2.0**24)
+            acc += int(s_int[r][g]) * (int(q_rows[r][j]) - int(z_rows[r][g])) * xi
+        out.append(acc)
+    return out
+
+
+def tolerance_rows_f64(Wd_rows, x16, K, rel: float = 2e-3) -> np.ndarray:
+    """rel * sum_{j in K} |W_ij| |x_j| for an fp64 weight (the dequantised one)."""
+    x = _as_f16(x16).reshape(-1)
+    Kl = np.asarray(K, dtype=np.int64)
+    return rel * (np.abs(np.asarray(Wd_rows, dtype=np.float64)[:, Kl]) @ np.abs(x[Kl].astype(np.float64)))
+
+
+def ref_pack_cmb_q(W16, bits: int):
+    """Bitmask packing with b-bit codes in place of the fp16 values.
+
+    Records are laid out as in :func:`ref_pack_cmb` (32 mask words, then the
+    stored entries in increasing row order, zero padding to 16 bytes), but an
+    entry is its code: one byte each for b = 8; for b = 4 two per byte, the
+    n-th entry of the record in byte n // 2, low nibble first when n is even.
+
+    The grids sit in a separate table of uint32 entries, s's fp16 bits in the
+    low half and z in the high half.  The entry of row i = 1024 s + 32 l + t
+    (segment s, lane l, bit t) and group g is at index
+    ((s * G + g) * 32 + t) * 32 + l; rows >= O hold 0.
+
+    Returns ``(header, off, data, table)``.
+    """
+    W = _as_f16(W16)
+    maxq = _check_bits(bits)
+    O, I = W.shape
+    S = (O + SEG_ROWS - 1) // SEG_ROWS
+    G = (I + QUANT_GROUP - 1) // QUANT_GROUP
+    q, s16, z = oracle_quantize_rtn(W, bits)
+    nzmask = (W.view(np.uint16) & 0x7FFF) != 0
+    off = np.zeros(I * S + 1, dtype=np.uint32)
+    pieces = []
+    pos = 0
+    nnz = 0
+    for j in range(I):
+        for s in range(S):
+            r0, r1 = s * SEG_ROWS, min(O, (s + 1) * SEG_ROWS)
+            m = np.zeros(SEG_ROWS, dtype=bool)
+            m[: r1 - r0] = nzmask[r0:r1, j]
+            codes = q[r0:r1, j][nzmask[r0:r1, j]]
+            assert codes.size == 0 or (codes.min() >= 0 and codes.max() <= maxq)
+            nnz += codes.size
+            if bits == 8:
+                cb = codes.astype(np.uint8).tobytes()
+            else:
+                nb = bytearray((codes.size + 1) // 2)
+                for n, c in enumerate(codes):
+                    nb[n // 2] |= int(c) << (4 * (n % 2))
+                cb = bytes(nb)
+            rec = np.packbits(m, bitorder="little").tobytes() + cb
+            rec = rec + b"\x00" * (_pad16(len(rec)) - len(rec))
+            off[j * S + s] = pos // 16
+            pos += len(rec)
+            pieces.append(rec)
+    off[I * S] = pos // 16
+    if pos // 16 >= 2**32:
+        raise ValueError("packed size exceeds the uint32 offset range")
+    data = np.frombuffer(b"".join(pieces), dtype=np.uint8).copy()
+    table = np.zeros(S * G * SEG_ROWS, dtype=np.uint32)
+    for s in range(S):
+        for g in range(G):
+            for t in range(32):
+                for l in range(32):
+                    i = s * SEG_ROWS + 32 * l + t
+                    if i < O:
+                        table[((s * G + g) * 32 + t) * 32 + l] = (
+                            int(s16[i, g].view(np.uint16)) | (int(z[i, g]) << 16))
+    header = dict(magic=CMB_MAGIC, version=CMB_VERSION, out=O, inp=I,
+                  seg_rows=SEG_ROWS, nseg=S, nnz=nnz, bits=bits, group=QUANT_GROUP)
+    return header, off, data, table
+
+
+def ref_unpack_cmb_q(header, off, data, table):
+    """Inverse of :func:`ref_pack_cmb_q`: returns ``(nz, q, s16, z)`` (the
+    non-zero mask O x I, the codes O x I with 0 where pruned, the grids)."""
+    O, I, S, bits = header["out"], header["inp"], header["nseg"], header["bits"]
+    G = (I + QUANT_GROUP - 1) // QUANT_GROUP
+    data = np.asarray(data, dtype=np.uint8)
+    nz = np.zeros((O, I), dtype=bool)
+    q = np.zeros((O, I), dtype=np.int64)
+    for j in range(I):
+        for s in range(S):
+            b0 = int(off[j * S + s]) * 16
+            words = np.frombuffer(data[b0:b0 + 128].tobytes(), dtype="<u4")
+            m = np.unpackbits(words.view(np.uint8), bitorder="little").astype(bool)
+            rows = np.nonzero(m)[0] + s * SEG_ROWS
+            if rows.size and rows[-1] >= O:
+                raise ValueError("mask bit set beyond the last row")
+            n = rows.size
+            cb = data[b0 + 128:b0 + 128 + (n if bits == 8 else (n + 1) // 2)]
+            if bits == 8:
+                codes = cb.astype(np.int64)
+            else:
+                codes = np.array([(int(cb[e // 2]) >> (4 * (e % 2))) & 15 for e in range(n)],
+                                 dtype=np.int64)
+            nz[rows, j] = True
+            q[rows, j] = codes
+    tab = np.asarray(table, dtype=np.uint32).reshape(S, G, 32, 32)   # [s][g][t][l]
+    rows_tab = tab.transpose(0, 3, 2, 1).reshape(S * SEG_ROWS, G)[:O]   # row 1024 s + 32 l + t
+    s16 = (rows_tab & 0xFFFF).astype(np.uint16).view(np.float16)
+    z = (rows_tab >> 16).astype(np.int64)
+    return nz, q, s16, z
+
+
+def required_bytes_q(nnz_per_channel, K, O: int, I: int, bits: int) -> float:
+    """Format-neutral bytes of a quantised call: b/8 bytes per stored entry of
+    the kept channels, one mask bit per (kept channel, row) position, an fp16
+    scale and a b-bit zero point per (row, group holding a kept channel), plus
+    x (2I), the kept ids and values (4k) and the fp32 output (4O)."""
+    _check_bits(bits)
+    n = np.asarray(nnz_per_channel, dtype=np.float64)
+    Kl = np.asarray(K, dtype=np.int64)
+    k = Kl.size
+    groups = np.unique(Kl // QUANT_GROUP).size
+    return float(bits / 8.0 * n[Kl].sum() + k * O / 8.0 + (2.0 + bits / 8.0) * O * groups
+                 + 2.0 * I + 4.0 * k + 4.0 * O)
