@@ -424,6 +424,7 @@ def run_ours(args):
             del gs
 
     thresh = run_threshold_path(duo, shape, layers, args.px, reps, peak)
+    quant = {f"int{b}": run_quant_path(duo, shape, layers, args.px, reps, peak, b) for b in (8, 4)}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -448,6 +449,7 @@ def run_ours(args):
             "dense_gemv_cublas": dense,
             "sweep_px": sweep,
             "threshold_path": thresh,
+            "quantised_values": quant,
         }
         print(json.dumps(line), flush=True)
     for lay in layers:
@@ -493,6 +495,59 @@ def run_threshold_path(duo, shape, layers, px, reps, peak):
     gbs = breq / (us * 1e-6) / 1e9
     return {"us_per_layer": us, "GB/s": gbs, "frac_of_peak": gbs / peak, "required_MB": breq / 1e6,
             "tau": "magnitude of the (k+1)-th largest |x| of each stage input, fixed before timing"}
+
+
+def run_quant_path(duo, shape, layers, px, reps, peak, bits):
+    """The same layer steps (fused top-k) over RTN-quantised stored values
+    (§5, weight-only quantisation with group size 128, Table 4): b-bit codes
+    in the records and one grid table per (segment, 128-channel group).
+    Required bytes: b/8 bytes per kept stored weight, one mask bit per kept
+    position, an fp16 scale and a b-bit zero point per (row, group holding a
+    kept channel), plus x, the kept list and y."""
+    L = len(layers)
+    fmt = "bitmask_q8" if bits == 8 else "bitmask_q4"
+    qh = [{p: duo.duo_pack(lay["W"][p], fmt) for p in lay["W"]} for lay in layers]
+    packed = sum(h.query().data_bytes + h.query().aux_bytes for h in qh[0].values())
+    breq = 0.0
+    for lay in layers:
+        for st, src in zip(STAGES, STAGE_SRC):
+            I = shape.I(st[0])
+            k = k_of(I, px)
+            groups = 0
+            if k > 0:
+                idx, _ = duo.duo_sparsify(lay["x"][src], k)
+                K = idx.to(torch.int64) & 0xFFFF
+                groups = int(torch.unique(K // 128).numel())
+            for p in st:
+                O = shape.O(p)
+                if k > 0:
+                    breq += (float(lay["nnz"][p][K].sum().item()) * bits / 8.0 + k * O / 8.0
+                             + (2.0 + bits / 8.0) * O * groups)
+                breq += 4.0 * O
+            breq += 2.0 * I + 4.0 * k
+    breq /= L
+
+    def fn():
+        for lay, hq in zip(layers, qh):
+            for st, src in zip(STAGES, STAGE_SRC):
+                k = k_of(shape.I(st[0]), px)
+                if len(st) == 1:
+                    duo.duo_spmspv(hq[st[0]], lay["x"][src], k, y=lay["y"][st[0]])
+                else:
+                    duo.duo_spmspv_multi([hq[p] for p in st], lay["x"][src], k,
+                                         ys=[lay["y"][p] for p in st])
+    g = capture(fn)
+    time_graph(g, 3)
+    r = max(3, min(reps, 500))
+    us = time_graph(g, r) / (r * L) * 1e6
+    del g
+    for hq in qh:
+        for h in hq.values():
+            h.free()
+    gbs = breq / (us * 1e-6) / 1e9
+    return {"us_per_layer": us, "GB/s": gbs, "frac_of_peak": gbs / peak, "required_MB": breq / 1e6,
+            "packed_MB_per_layer": packed / 1e6, "bits": bits, "group": 128,
+            "grid": "asymmetric min-max per (row, 128-channel group), fp16 scale, RTN"}
 
 
 def run_e2e(duo, shape, layers, args, breq_mean):

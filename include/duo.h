@@ -52,9 +52,12 @@ enum {
 /* Packed weight formats (the paper fixes none: §4.1 only says each weight
  * column is stored compressed; both layouts below are this library's). */
 enum {
-    DUO_FMT_IDX16 = 0,   /* per channel: fp16 non-zeros + uint16 row ids */
-    DUO_FMT_BITMASK = 1  /* "CMB": per (channel, 1024-row segment) a 128-byte
-                            row bitmask followed by the fp16 non-zeros */
+    DUO_FMT_IDX16 = 0,      /* per channel: fp16 non-zeros + uint16 row ids */
+    DUO_FMT_BITMASK = 1,    /* "CMB": per (channel, 1024-row segment) a 128-byte
+                               row bitmask followed by the fp16 non-zeros */
+    DUO_FMT_BITMASK_Q8 = 2, /* CMB with 8-bit RTN codes in place of the fp16
+                               non-zeros, plus a table of grids (see duo_pack) */
+    DUO_FMT_BITMASK_Q4 = 3  /* the same with 4-bit codes, two per byte */
 };
 
 /* Opaque packed weight, owned by the library from duo_pack to duo_free. */
@@ -70,7 +73,8 @@ typedef struct duo_packed duo_packed;
  *                -0 are pruned, every other entry is stored bit-exactly.
  *   out, in    : O >= 1 and 1 <= I <= 65535; IDX16 also needs O <= 65536.
  *   ldw        : >= in.
- *   fmt        : DUO_FMT_BITMASK or DUO_FMT_IDX16.
+ *   fmt        : DUO_FMT_BITMASK, DUO_FMT_BITMASK_Q8, DUO_FMT_BITMASK_Q4 or
+ *                DUO_FMT_IDX16.
  *   stream     : work is enqueued on it and the call synchronises it before
  *                returning (the packed size must be known to allocate).
  *   h_out      : receives the new handle; untouched on error.
@@ -81,6 +85,20 @@ typedef struct duo_packed duo_packed;
  * iff W[s*1024 + 32*w + b, j] != 0; rows >= O give 0), then those entries'
  * fp16 bit patterns in increasing row order, zero padded to 16 bytes.
  * off is uint32[I*S + 1]; off[I*S] is the total size in 16-byte units.
+ *
+ * BITMASK_Q8 / _Q4 layout (§5, weight-only quantisation with channel-wise
+ * RTN and group size 128, Table 4; the grid is this library's reading of it):
+ * each (row i, group g of input channels 128g .. 128g+127) has the
+ * asymmetric min-max grid lo = min(0, min W), hi = max(0, max W) over the
+ * group's stored weights, s = fp16((hi - lo) / (2^b - 1)) from an fp64
+ * quotient (1 if the group stores nothing, 2^-24 if the quotient rounds to
+ * 0), z = rint(-lo / s) clamped to [0, 2^b - 1]; a stored weight w becomes
+ * q = clamp(rint(w / s) + z, 0, 2^b - 1) (fp64 quotient, ties to even) and
+ * stands for s (q - z).  Records are as for BITMASK with the codes in place
+ * of the fp16 values: one byte each (Q8) or two per byte, the n-th code of
+ * the record in byte n / 2, low nibble first (Q4).  The grids are the aux
+ * buffer: uint32 entries s_bits | z << 16, entry ((s * G + g) * 32 + t) * 32
+ * + l for row i = 1024 s + 32 l + t, G = ceil(I / 128); rows >= O hold 0.
  *
  * IDX16 layout: per channel j a block at byte colptr[j]: cnt[j] fp16
  * non-zeros (increasing row), zero padded to 16 bytes, then their uint16 row
@@ -116,11 +134,19 @@ int duo_sparsify(const void* x_fp16_dev, int64_t in, int64_t k,
  *             compressed columns.
  *   listed  : kept_idx_dev (uint16[k], distinct ids < in, any order) and
  *             kept_val_fp16_dev (fp16[k]) give the sparse input directly;
- *             x_fp16_dev is ignored and may be NULL.
+ *             x_fp16_dev is ignored and may be NULL.  For BITMASK_Q8 / _Q4
+ *             handles the ids must not decrease in id / 128 (ascending ids
+ *             do); a list out of that order is rejected on the device
+ *             (duo_device_status then returns DUO_EFORMAT).
+ *   coded   : BITMASK_Q8 / _Q4 handles need every (handle, 1024-row
+ *             segment) pair of the call to have an SM of its own (at most
+ *             one per SM of the device, e.g. 152 on a GB300): DUO_ERANGE
+ *             otherwise.  y sums the dequantised weights s (q - z).
  *   k == 0  : y = 0; the input pointers are not read and may be NULL.
  *   y_dev   : device fp32[O], 16-byte aligned; fully overwritten.  Summation
  *             order is not fixed, so y is reproducible only to fp32 rounding.
- * Errors: DUO_EINVAL (NULL, alignment, k, dead handle), DUO_ECUDA.
+ * Errors: DUO_EINVAL (NULL, alignment, k, dead handle), DUO_ERANGE,
+ * DUO_ECUDA.
  */
 /* Concurrency: calls whose first handle is the same must be ordered on the
  * GPU (same stream, or otherwise synchronised): the bitmask kernel keeps a
@@ -183,6 +209,8 @@ int duo_free(duo_packed* h);
 
 /* Describes a live handle.  Pointers stay owned by the handle.
  *   BITMASK: index = uint32 off[I*S+1], aux = NULL.
+ *   BITMASK_Q8 / _Q4: index = uint32 off[I*S+1], aux = uint32 grids
+ *            [S][ceil(I/128)][1024] (layout under duo_pack).
  *   IDX16  : index = uint64 colptr[I+1], aux = uint32 cnt[I]. */
 typedef struct duo_packed_info {
     int32_t fmt;

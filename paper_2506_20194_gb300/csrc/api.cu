@@ -30,6 +30,7 @@ struct duo_packed {
   int64_t aux_bytes;
   void* data;
   int64_t data_bytes;
+  int vbits;           // BITMASK formats: bits per stored value (16, 8, 4)
   unsigned int* sync;  // BITMASK: 2-word grid barrier of the spMspV kernel
   uint16_t* kept;      // BITMASK: room for a kept list (ids, then values; 2 x in each)
   int max_record;      // BITMASK: bytes of the largest record
@@ -81,6 +82,14 @@ cudaError_t duo_malloc(void** p, size_t bytes) {
 }
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+bool is_cmb(int fmt) {
+  return fmt == DUO_FMT_BITMASK || fmt == DUO_FMT_BITMASK_Q8 || fmt == DUO_FMT_BITMASK_Q4;
+}
+
+int fmt_vbits(int fmt) {
+  return fmt == DUO_FMT_BITMASK_Q8 ? 8 : (fmt == DUO_FMT_BITMASK_Q4 ? 4 : 16);
+}
 
 // True if p is device (or managed) memory of the current context.
 bool is_device_ptr(const void* p) {
@@ -138,7 +147,7 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
              duo_packed** h_out) {
   if (W_fp16_dev == nullptr || h_out == nullptr) return DUO_EINVAL;
   if (out < 1 || in < 1 || ldw < in) return DUO_EINVAL;
-  if (fmt != DUO_FMT_IDX16 && fmt != DUO_FMT_BITMASK) return DUO_EINVAL;
+  if (fmt != DUO_FMT_IDX16 && !is_cmb(fmt)) return DUO_EINVAL;
   if (!aligned(W_fp16_dev, 2)) return DUO_EINVAL;
   if (in > 65535) return DUO_ERANGE;
   if (fmt == DUO_FMT_IDX16 && out > 65536) return DUO_ERANGE;
@@ -166,6 +175,7 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
   duo_packed* h = new (std::nothrow) duo_packed();
   if (h == nullptr) return DUO_ENOMEM;
   h->fmt = fmt;
+  h->vbits = fmt_vbits(fmt);
   h->out = out;
   h->in = in;
   cudaGetDevice(&h->device);
@@ -181,8 +191,19 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
   };
 
   unsigned long long host_tot[3] = {0, 0, 0};
-  if (fmt == DUO_FMT_BITMASK) {
+  if (is_cmb(fmt)) {
     h->nseg = S;
+    if (h->vbits < 16) {
+      // Grid tables first: the scatter reads them to code the weights.
+      const int64_t G = (in + 127) / 128;
+      h->aux_bytes = (int64_t)sizeof(uint32_t) * S * G * duo::kSegRows;
+      e = duo_malloc(&aux, (size_t)h->aux_bytes);
+      if (e != cudaSuccess) return fail(map_err(e));
+      e = cudaMemsetAsync(aux, 0, (size_t)h->aux_bytes, st);
+      if (e != cudaSuccess) return fail(map_err(e));
+      e = duo::launch_quant_grid(W, out, in, ldw, (int)S, h->vbits, static_cast<uint32_t*>(aux), st);
+      if (e != cudaSuccess) return fail(map_err(e));
+    }
     h->index_bytes = (int64_t)sizeof(uint32_t) * (in * S + 1);
     // The offsets are followed (at a 256-byte boundary) by the two barrier
     // words of the spMspV kernel, zeroed here.
@@ -195,20 +216,20 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
     h->kept = reinterpret_cast<uint16_t*>(static_cast<char*>(index) + sync_at + 256);
     e = cudaMemsetAsync(h->sync, 0, 256, st);
     if (e != cudaSuccess) return fail(map_err(e));
-    e = duo::launch_cmb_offsets(cnt_js, in * S, static_cast<uint32_t*>(index), totals, st);
+    e = duo::launch_cmb_offsets(cnt_js, in * S, h->vbits, static_cast<uint32_t*>(index), totals, st);
     if (e != cudaSuccess) return fail(map_err(e));
     e = cudaMemcpyAsync(host_tot, totals, sizeof(host_tot), cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return fail(map_err(e));
     if (host_tot[0] >= (1ull << 32)) return fail(DUO_ERANGE);
     h->data_bytes = (int64_t)host_tot[0] * 16;
-    h->max_record = (int)((128 + 2 * host_tot[2] + 15) / 16 * 16);
+    h->max_record = (int)((128 + (host_tot[2] * h->vbits + 7) / 8 + 15) / 16 * 16);
     e = duo_malloc(&data, (size_t)h->data_bytes);
     if (e != cudaSuccess) return fail(map_err(e));
     e = cudaMemsetAsync(data, 0, (size_t)h->data_bytes, st);
     if (e != cudaSuccess) return fail(map_err(e));
-    e = duo::launch_cmb_scatter(W, out, in, ldw, (int)S, static_cast<const uint32_t*>(index),
-                                static_cast<uint8_t*>(data), st);
+    e = duo::launch_cmb_scatter(W, out, in, ldw, (int)S, h->vbits, static_cast<const uint32_t*>(aux),
+                                static_cast<const uint32_t*>(index), static_cast<uint8_t*>(data), st);
     if (e != cudaSuccess) return fail(map_err(e));
   } else {
     h->nseg = 0;
@@ -292,7 +313,7 @@ int duo_spmspv_threshold(const duo_packed* const* hs, int n, const void* x_fp16_
   for (int p = 0; p < n; ++p) {
     if (hs[p] == nullptr || ys_dev[p] == nullptr || !aligned(ys_dev[p], 16)) return DUO_EINVAL;
     if (!is_live(hs[p])) return DUO_EINVAL;
-    if (hs[p]->fmt != DUO_FMT_BITMASK) return DUO_EFORMAT;
+    if (!is_cmb(hs[p]->fmt) || hs[p]->fmt != hs[0]->fmt) return DUO_EFORMAT;
     if (hs[p]->in != hs[0]->in) return DUO_EINVAL;
   }
   int rc = cuda_ready();
@@ -306,6 +327,7 @@ int duo_spmspv_threshold(const duo_packed* const* hs, int n, const void* x_fp16_
   a.kval = nullptr;
   a.thresh = 1;
   a.tau_key = tau_fp16 & 0x7FFFu;
+  a.vbits = hs[0]->vbits;
   a.bar = hs[0]->sync;
   a.slot_bytes = 0;
   for (int p = 0; p < n; ++p) {
@@ -315,6 +337,8 @@ int duo_spmspv_threshold(const duo_packed* const* hs, int n, const void* x_fp16_
     a.p[p].y = ys_dev[p];
     a.p[p].O = (int)hs[p]->out;
     a.p[p].S = (int)hs[p]->nseg;
+    a.p[p].G = (int)((hs[p]->in + 127) / 128);
+    a.p[p].qtab = static_cast<const uint32_t*>(hs[p]->aux);
     a.p[p].dens = (float)((double)hs[p]->nnz / ((double)hs[p]->out * (double)hs[p]->in));
   }
   cudaError_t e = duo::launch_cmb_spmspv(a, static_cast<cudaStream_t>(stream));
@@ -339,14 +363,14 @@ static int spmspv_common(const duo_packed* const* hs, int n, const void* x, cons
   const int64_t I = hs[0]->in;
   for (int p = 1; p < n; ++p) {
     if (hs[p]->in != I) return DUO_EINVAL;
-    if (hs[p]->fmt != DUO_FMT_BITMASK) return DUO_EFORMAT;
+    if (!is_cmb(hs[p]->fmt) || hs[p]->fmt != hs[0]->fmt) return DUO_EFORMAT;
   }
-  if (n > 1 && hs[0]->fmt != DUO_FMT_BITMASK) return DUO_EFORMAT;
+  if (n > 1 && !is_cmb(hs[0]->fmt)) return DUO_EFORMAT;
   if (k < 0 || k > I) return DUO_EINVAL;
   int rc = cuda_ready();
   if (rc != DUO_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (k == 0 || hs[0]->fmt != DUO_FMT_BITMASK) {
+  if (k == 0 || !is_cmb(hs[0]->fmt)) {
     // The bitmask kernel zeroes y itself; other paths clear it here.
     for (int p = 0; p < n; ++p) {
       cudaError_t e = cudaMemsetAsync(ys[p], 0, sizeof(float) * (size_t)hs[p]->out, st);
@@ -355,11 +379,12 @@ static int spmspv_common(const duo_packed* const* hs, int n, const void* x, cons
   }
   if (k == 0) return DUO_OK;
   cudaError_t e;
-  if (hs[0]->fmt == DUO_FMT_BITMASK) {
+  if (is_cmb(hs[0]->fmt)) {
     duo::CmbArgs a{};
     a.np = n;
     a.I = (int)I;
     a.k = (int)k;
+    a.vbits = hs[0]->vbits;
     a.x = static_cast<const uint16_t*>(x);
     a.kidx = listed ? kidx : nullptr;
     a.kval = listed ? static_cast<const uint16_t*>(kval) : nullptr;
@@ -372,6 +397,8 @@ static int spmspv_common(const duo_packed* const* hs, int n, const void* x, cons
       a.p[p].y = ys[p];
       a.p[p].O = (int)hs[p]->out;
       a.p[p].S = (int)hs[p]->nseg;
+      a.p[p].G = (int)((hs[p]->in + 127) / 128);
+      a.p[p].qtab = static_cast<const uint32_t*>(hs[p]->aux);
       a.p[p].dens = (float)((double)hs[p]->nnz / ((double)hs[p]->out * (double)hs[p]->in));
     }
     e = duo::launch_cmb_spmspv(a, st);
@@ -441,9 +468,9 @@ int duo_packed_query(const duo_packed* h, duo_packed_info* info) {
   if (h == nullptr || info == nullptr || !is_live(h)) return DUO_EINVAL;
   std::memset(info, 0, sizeof(*info));
   info->fmt = h->fmt;
-  info->version = h->fmt == DUO_FMT_BITMASK ? 1 : 0;
-  info->magic = h->fmt == DUO_FMT_BITMASK ? kCmbMagic : kIdx16Magic;
-  info->seg_rows = h->fmt == DUO_FMT_BITMASK ? duo::kSegRows : 0;
+  info->version = is_cmb(h->fmt) ? 1 : 0;
+  info->magic = is_cmb(h->fmt) ? kCmbMagic : kIdx16Magic;
+  info->seg_rows = is_cmb(h->fmt) ? duo::kSegRows : 0;
   info->out = h->out;
   info->in = h->in;
   info->nseg = h->nseg;

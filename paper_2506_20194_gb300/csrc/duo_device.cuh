@@ -202,6 +202,55 @@ __device__ __forceinline__ float fma_f16_f32(uint16_t w, uint16_t x, float acc) 
   return acc;
 }
 
+// ---- Quantised values (§5, weight-only quantisation, Table 4) ----
+// A b-bit code q of row i in input-channel group g (128 channels) stands for
+// s (q - z), with {fp16 s, z} the grid of (i, g).  Grid tables hold one
+// (segment, group) each: entry 32 t + l is row 32 l + t of the segment.
+constexpr int QGROUP = 128;                    // input channels per grid
+constexpr int QTAB_BYTES = SEG_ROWS * 4;       // one table: 1024 uint32 entries
+constexpr int QNTB = 4;                        // tables a CTA holds at once
+
+// Walk over one lane's codes in a record, from its first code on.  at()
+// reads the code at the current position whether or not the row has one
+// (the byte after a lane's last code is still inside the record's slot or
+// the 16 bytes of slack after the ring), and step(bit) moves on by one code
+// when bit is 1: no branch per row.
+template <int VB>
+struct CodeWalk;
+
+template <>
+struct CodeWalk<8> {   // one byte per code
+  const uint8_t* p;
+  __device__ __forceinline__ void init(const uint8_t* codes, uint32_t first) { p = codes + first; }
+  __device__ __forceinline__ uint32_t at() const { return *p; }
+  __device__ __forceinline__ void step(uint32_t bit) { p += bit; }
+};
+
+template <>
+struct CodeWalk<4> {   // two codes per byte, the even one in the low nibble
+  const uint8_t* p;
+  uint32_t sh;
+  __device__ __forceinline__ void init(const uint8_t* codes, uint32_t first) {
+    p = codes + (first >> 1);
+    sh = (first & 1u) << 2;
+  }
+  __device__ __forceinline__ uint32_t at() const { return ((uint32_t)*p >> sh) & 15u; }
+  __device__ __forceinline__ void step(uint32_t bit) {
+    p += (sh >> 2) & bit;
+    sh ^= bit << 2;
+  }
+};
+
+// acc + bit * s (q - z) x (bit 0 or 1, no branch), with e = s's fp16 bits |
+// z << 16 (z <= 255): q - z is the exact difference of 2^23 + q and
+// 2^23 + z, s x is exact in fp32 (fp16 x fp16), and the fma rounds once.
+__device__ __forceinline__ float q_fma_sel(uint32_t bit, uint32_t q, uint32_t e, uint16_t x, float acc) {
+  const float d = __uint_as_float(0x4B000000u | q) -
+                  __uint_as_float(__byte_perm(e, 0x4B000000u, 0x7542));
+  const float sx = fma_f16_f32((uint16_t)(e & 0xFFFFu), x, 0.f);
+  return fmaf(bit ? d : 0.f, sx, acc);
+}
+
 __device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, float d) {
   asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c),
                "f"(d)

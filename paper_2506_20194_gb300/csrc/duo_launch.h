@@ -21,8 +21,10 @@ struct CmbProb {
   const uint8_t* data;   // records
   const uint32_t* off;   // off[I*S + 1], 16-byte units
   float* y;              // fp32[O], zeroed before the launch
+  const uint32_t* qtab;  // quantised formats: grid tables [S][G][1024] ({fp16 s, z})
   int O;
   int S;
+  int G;                 // quantised formats: input-channel groups ceil(I / 128)
   float dens;            // non-zeros / (O * I): to estimate record sizes
 };
 
@@ -43,6 +45,7 @@ struct CmbArgs {
   int list_cap;          // set by the launcher: kept-list entries a CTA emits
   int thresh;            // in: 1 = threshold mask (keep key > tau_key), 0 = top-k / listed
   uint32_t tau_key;      // in: threshold as an fp16 magnitude bit pattern (bits & 0x7FFF)
+  int vbits;             // in: bits of a stored value: 16 (fp16), 8 or 4 (RTN codes)
   int nruns;             // set by the launcher: > 0 when each (problem, segment)
                          // run has CTAs of its own: run r (items r*k .. r*k+k-1)
                          // goes to CTAs run_cta[r] .. run_cta[r+1]-1
@@ -76,13 +79,19 @@ cudaError_t launch_sparsify(const uint16_t* x, int I, int k, uint16_t* kidx, uin
 // Packing.  cnt_js[j*S + s] = non-zeros of channel j in row segment s.
 cudaError_t launch_pack_count(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
                               uint32_t* cnt_js, cudaStream_t st);
-// off[n] exclusive prefix (16-byte units) of the CMB record sizes;
-// totals[0] = total units (64-bit), totals[1] = total non-zeros,
-// totals[2] = largest per-record non-zero count.
-cudaError_t launch_cmb_offsets(const uint32_t* cnt_js, int64_t n, uint32_t* off,
+// off[n] exclusive prefix (16-byte units) of the CMB record sizes for
+// vbits-bit values (16, 8 or 4); totals[0] = total units (64-bit),
+// totals[1] = total non-zeros, totals[2] = largest per-record non-zero count.
+cudaError_t launch_cmb_offsets(const uint32_t* cnt_js, int64_t n, int vbits, uint32_t* off,
                                unsigned long long* totals, cudaStream_t st);
+// RTN grids of every (row, 128-channel group) into table[S][G][1024]
+// (zeroed by the caller; rows >= O stay 0).
+cudaError_t launch_quant_grid(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S, int bits,
+                              uint32_t* table, cudaStream_t st);
+// Records: fp16 values (vbits 16) or the codes of the grids in table.
 cudaError_t launch_cmb_scatter(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
-                               const uint32_t* off, uint8_t* data, cudaStream_t st);
+                               int vbits, const uint32_t* table, const uint32_t* off,
+                               uint8_t* data, cudaStream_t st);
 // cnt[j] = sum_s cnt_js, colptr[j] byte offsets of the IDX16 blocks;
 // totals[0] = total bytes, totals[1] = total non-zeros.
 cudaError_t launch_idx16_offsets(const uint32_t* cnt_js, int64_t I, int S, uint32_t* cnt,

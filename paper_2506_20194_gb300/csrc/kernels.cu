@@ -50,6 +50,8 @@ __host__ __device__ inline size_t align_up(size_t v, size_t a) { return (v + a -
 constexpr int PACK_THREADS = 256;
 constexpr int PACK_PITCH = 34;  // halves per tile row
 constexpr size_t PACK_SMEM = (size_t)SEG_ROWS * PACK_PITCH * 2;
+constexpr int QT_PITCH = 33;    // uint32 per row of a grid table staged for the scatter
+constexpr size_t PACK_QSMEM = PACK_SMEM + (size_t)32 * QT_PITCH * 4;
 
 enum PackMode { PACK_COUNT = 0, PACK_CMB = 1, PACK_IDX16 = 2 };
 
@@ -62,10 +64,21 @@ struct PackArgs {
   const uint32_t* off;       // CMB
   const uint32_t* cnt;       // IDX16
   const uint64_t* colptr;    // IDX16
+  const uint32_t* qtab;      // CMB, VB < 16: grid tables
+  int G;                     // CMB, VB < 16: input-channel groups
   uint8_t* data;
 };
 
-template <int MODE>
+// RTN code of a stored weight w (fp16 bits) on the grid e = {fp16 s, z}
+// (§5, weight-only quantisation): clamp(rint(w / s) + z, 0, maxq), the
+// quotient in fp64.
+__device__ __forceinline__ uint32_t rtn_code(uint16_t w, uint32_t e, int maxq) {
+  const double s = (double)__half2float(__ushort_as_half((unsigned short)(e & 0xFFFFu)));
+  const double q = rint((double)__half2float(__ushort_as_half(w)) / s) + (double)(e >> 16);
+  return (uint32_t)fmin(fmax(q, 0.0), (double)maxq);
+}
+
+template <int MODE, int VB>
 __global__ void __launch_bounds__(PACK_THREADS) pack_tile_kernel(const PackArgs a) {
   extern __shared__ __align__(16) uint16_t tile[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -76,11 +89,20 @@ __global__ void __launch_bounds__(PACK_THREADS) pack_tile_kernel(const PackArgs 
   const int rows = rows64 < SEG_ROWS ? (int)rows64 : SEG_ROWS;
   const int64_t ncol64 = a.I - j0;
   const int ncol = ncol64 < 32 ? (int)ncol64 : 32;
+  constexpr bool QUANT = MODE == PACK_CMB && VB < 16;
+  uint32_t* qs = reinterpret_cast<uint32_t*>(tile + (size_t)SEG_ROWS * PACK_PITCH);
   for (int e = tid; e < SEG_ROWS * 32; e += PACK_THREADS) {
     const int r = e >> 5, c = e & 31;
     uint16_t v = 0;
     if (r < rows && c < ncol) v = a.W[(r0 + r) * a.ldw + j0 + c];
     tile[r * PACK_PITCH + c] = v;
+  }
+  if (QUANT) {
+    // The grid table of (segment s, group j0 / 128): the 32 channels of the
+    // tile share it.  Entry 32 b + t (row 32 t + b) goes to qs[b * 33 + t],
+    // so the walk below (lane b, word t) reads distinct banks.
+    const uint32_t* src = a.qtab + ((size_t)s * a.G + (size_t)(j0 / QGROUP)) * SEG_ROWS;
+    for (int e = tid; e < SEG_ROWS; e += PACK_THREADS) qs[(e >> 5) * QT_PITCH + (e & 31)] = src[e];
   }
   __syncthreads();
   const uint32_t lt = (1u << lane) - 1u;
@@ -88,10 +110,13 @@ __global__ void __launch_bounds__(PACK_THREADS) pack_tile_kernel(const PackArgs 
     const int64_t j = j0 + c;
     uint32_t total = 0, myword = 0;
     uint16_t* vals = nullptr;
+    uint8_t* codes = nullptr;
     uint16_t* rowids = nullptr;
+    uint32_t pend = 0;   // VB == 4: the code waiting for its byte's high nibble
     if (MODE == PACK_CMB) {
       const uint32_t o = a.off[j * a.S + s];
       vals = reinterpret_cast<uint16_t*>(a.data + (size_t)o * 16 + MASK_BYTES);
+      codes = a.data + (size_t)o * 16 + MASK_BYTES;
     } else if (MODE == PACK_IDX16) {
       uint32_t pre = 0;
       for (int s2 = 0; s2 < s; ++s2) pre += a.cnt_js_in[j * a.S + s2];
@@ -107,7 +132,24 @@ __global__ void __launch_bounds__(PACK_THREADS) pack_tile_kernel(const PackArgs 
       const uint32_t word = __ballot_sync(FULL_MASK, nz);
       if (MODE == PACK_CMB) {
         if (lane == t) myword = word;
-        if (nz) vals[total + __popc(word & lt)] = v;
+        const uint32_t pos = total + __popc(word & lt);
+        if (VB == 16) {
+          if (nz) vals[pos] = v;
+        } else {
+          const uint32_t q = nz ? rtn_code(v, qs[lane * QT_PITCH + t], (1 << VB) - 1) : 0u;
+          if (VB == 8) {
+            if (nz) codes[pos] = (uint8_t)q;
+          } else {
+            // Code n goes to byte n / 2, low nibble when n is even.  A lane
+            // at an odd position writes its byte with the code before it:
+            // the previous set lane's, or the word's carried-over last code.
+            const uint32_t below = word & lt;
+            const int prev = below ? 31 - __clz(below) : lane;
+            const uint32_t qprev = __shfl_sync(FULL_MASK, q, prev);
+            if (nz && (pos & 1u)) codes[pos >> 1] = (uint8_t)((below ? qprev : pend) | (q << 4));
+            if (word != 0u) pend = __shfl_sync(FULL_MASK, q, 31 - __clz(word));
+          }
+        }
       } else if (MODE == PACK_IDX16) {
         if (nz) {
           const uint32_t pos = total + __popc(word & lt);
@@ -122,33 +164,19 @@ __global__ void __launch_bounds__(PACK_THREADS) pack_tile_kernel(const PackArgs 
     } else if (MODE == PACK_CMB) {
       const uint32_t o = a.off[j * a.S + s];
       reinterpret_cast<uint32_t*>(a.data + (size_t)o * 16)[lane] = myword;
+      if (VB == 4 && (total & 1u) && lane == 0) codes[total >> 1] = (uint8_t)pend;
     }
   }
 }
 
-static cudaError_t launch_pack_tiles(int mode, const PackArgs& a, cudaStream_t st) {
+template <int MODE, int VB>
+static cudaError_t launch_pack_tiles_t(const PackArgs& a, cudaStream_t st) {
   const dim3 grid((unsigned)((a.I + 31) / 32), (unsigned)a.S);
-  cudaError_t e;
-  switch (mode) {
-    case PACK_COUNT:
-      e = cudaFuncSetAttribute(pack_tile_kernel<PACK_COUNT>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PACK_SMEM);
-      if (e != cudaSuccess) return e;
-      pack_tile_kernel<PACK_COUNT><<<grid, PACK_THREADS, PACK_SMEM, st>>>(a);
-      break;
-    case PACK_CMB:
-      e = cudaFuncSetAttribute(pack_tile_kernel<PACK_CMB>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PACK_SMEM);
-      if (e != cudaSuccess) return e;
-      pack_tile_kernel<PACK_CMB><<<grid, PACK_THREADS, PACK_SMEM, st>>>(a);
-      break;
-    default:
-      e = cudaFuncSetAttribute(pack_tile_kernel<PACK_IDX16>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PACK_SMEM);
-      if (e != cudaSuccess) return e;
-      pack_tile_kernel<PACK_IDX16><<<grid, PACK_THREADS, PACK_SMEM, st>>>(a);
-      break;
-  }
+  const size_t smem = (MODE == PACK_CMB && VB < 16) ? PACK_QSMEM : PACK_SMEM;
+  cudaError_t e = cudaFuncSetAttribute(pack_tile_kernel<MODE, VB>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  pack_tile_kernel<MODE, VB><<<grid, PACK_THREADS, smem, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -156,14 +184,22 @@ cudaError_t launch_pack_count(const uint16_t* W, int64_t O, int64_t I, int64_t l
                               uint32_t* cnt_js, cudaStream_t st) {
   PackArgs a{};
   a.W = W; a.O = O; a.I = I; a.ldw = ldw; a.S = S; a.cnt_js = cnt_js;
-  return launch_pack_tiles(PACK_COUNT, a, st);
+  return launch_pack_tiles_t<PACK_COUNT, 16>(a, st);
 }
 
 cudaError_t launch_cmb_scatter(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
-                               const uint32_t* off, uint8_t* data, cudaStream_t st) {
+                               int vbits, const uint32_t* table, const uint32_t* off,
+                               uint8_t* data, cudaStream_t st) {
   PackArgs a{};
   a.W = W; a.O = O; a.I = I; a.ldw = ldw; a.S = S; a.off = off; a.data = data;
-  return launch_pack_tiles(PACK_CMB, a, st);
+  a.qtab = table;
+  a.G = (int)((I + QGROUP - 1) / QGROUP);
+  switch (vbits) {
+    case 16: return launch_pack_tiles_t<PACK_CMB, 16>(a, st);
+    case 8: return launch_pack_tiles_t<PACK_CMB, 8>(a, st);
+    case 4: return launch_pack_tiles_t<PACK_CMB, 4>(a, st);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 cudaError_t launch_idx16_scatter(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S,
@@ -172,7 +208,66 @@ cudaError_t launch_idx16_scatter(const uint16_t* W, int64_t O, int64_t I, int64_
   PackArgs a{};
   a.W = W; a.O = O; a.I = I; a.ldw = ldw; a.S = S; a.cnt_js_in = cnt_js; a.cnt = cnt;
   a.colptr = colptr; a.data = data;
-  return launch_pack_tiles(PACK_IDX16, a, st);
+  return launch_pack_tiles_t<PACK_IDX16, 16>(a, st);
+}
+
+// RTN grids (§5, weight-only quantisation with channel-wise RTN, group size
+// 128): one warp per (row i, group g), lanes covering four channels each.
+// lo = min(0, min w), hi = max(0, max w) over the group's stored weights;
+// s = fp16((hi - lo) / maxq) from an fp64 quotient (1 for an empty group,
+// 2^-24 if it rounds to 0); z = rint(-lo / s) clamped to [0, maxq].
+constexpr int QGRID_THREADS = 256;
+
+__global__ void __launch_bounds__(QGRID_THREADS) quant_grid_kernel(const uint16_t* __restrict__ W,
+                                                                    int64_t O, int64_t I, int64_t ldw,
+                                                                    int G, int maxq,
+                                                                    uint32_t* __restrict__ table) {
+  const int lane = threadIdx.x & 31;
+  const int64_t wg = (int64_t)blockIdx.x * (QGRID_THREADS / 32) + (threadIdx.x >> 5);
+  if (wg >= O * G) return;   // whole warps
+  const int64_t i = wg / G;
+  const int g = (int)(wg - i * G);
+  float lo = 0.f, hi = 0.f;   // fp16 values are exact in fp32
+  for (int e = lane; e < QGROUP; e += 32) {
+    const int64_t j = (int64_t)g * QGROUP + e;
+    if (j < I) {
+      const uint16_t b = W[i * ldw + j];
+      if (b & 0x7FFFu) {
+        const float v = __half2float(__ushort_as_half(b));
+        lo = fminf(lo, v);
+        hi = fmaxf(hi, v);
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lo = fminf(lo, __shfl_xor_sync(FULL_MASK, lo, o));
+    hi = fmaxf(hi, __shfl_xor_sync(FULL_MASK, hi, o));
+  }
+  if (lane == 0) {
+    uint32_t sb = 0x3C00u;
+    if (hi != lo) {
+      sb = __half_as_ushort(__double2half(((double)hi - (double)lo) / (double)maxq));
+      if (sb == 0u) sb = 1u;
+    }
+    const double sd = (double)__half2float(__ushort_as_half((unsigned short)sb));
+    const double zd = fmin(fmax(rint(-(double)lo / sd), 0.0), (double)maxq);
+    const int64_t seg = i / SEG_ROWS, r = i - seg * SEG_ROWS;
+    table[((seg * G + g) * 32 + (r & 31)) * 32 + (r >> 5)] = sb | ((uint32_t)zd << 16);
+  }
+}
+
+cudaError_t launch_quant_grid(const uint16_t* W, int64_t O, int64_t I, int64_t ldw, int S, int bits,
+                              uint32_t* table, cudaStream_t st) {
+  (void)S;
+  if (bits != 8 && bits != 4) return cudaErrorInvalidValue;
+  const int64_t G = (I + QGROUP - 1) / QGROUP;
+  const int64_t warps = O * G;
+  const int64_t blocks = (warps + QGRID_THREADS / 32 - 1) / (QGRID_THREADS / 32);
+  if (blocks > 0x7FFFFFFF) return cudaErrorInvalidValue;
+  quant_grid_kernel<<<(unsigned)blocks, QGRID_THREADS, 0, st>>>(W, O, I, ldw, (int)G, (1 << bits) - 1,
+                                                               table);
+  return cudaGetLastError();
 }
 
 // Single-CTA chunked exclusive scan (packing is an offline step; one CTA
@@ -228,11 +323,11 @@ __device__ void chunked_scan(int64_t n, F value, G emit, unsigned long long* tot
 }
 
 __global__ void __launch_bounds__(SCAN_THREADS) cmb_offsets_kernel(const uint32_t* cnt_js, int64_t n,
-                                                                   uint32_t* off,
+                                                                   int vbits, uint32_t* off,
                                                                    unsigned long long* totals) {
-  // record units = (128 + pad16(2 * cnt)) / 16 = 8 + ceil(cnt / 8)
+  // record units = (128 + pad16(ceil(cnt * vbits / 8))) / 16 = 8 + ceil(cnt * vbits / 128)
   chunked_scan(
-      n, [&](int64_t i) { return 8ull + (cnt_js[i] + 7ull) / 8ull; },
+      n, [&](int64_t i) { return 8ull + ((unsigned long long)cnt_js[i] * vbits + 127ull) / 128ull; },
       [&](int64_t i, unsigned long long pre) { off[i] = (uint32_t)pre; }, &totals[0]);
   __syncthreads();
   chunked_scan(
@@ -253,9 +348,10 @@ __global__ void __launch_bounds__(SCAN_THREADS) cmb_offsets_kernel(const uint32_
   }
 }
 
-cudaError_t launch_cmb_offsets(const uint32_t* cnt_js, int64_t n, uint32_t* off,
+cudaError_t launch_cmb_offsets(const uint32_t* cnt_js, int64_t n, int vbits, uint32_t* off,
                                unsigned long long* totals, cudaStream_t st) {
-  cmb_offsets_kernel<<<1, SCAN_THREADS, 0, st>>>(cnt_js, n, off, totals);
+  if (vbits != 16 && vbits != 8 && vbits != 4) return cudaErrorInvalidValue;
+  cmb_offsets_kernel<<<1, SCAN_THREADS, 0, st>>>(cnt_js, n, vbits, off, totals);
   return cudaGetLastError();
 }
 
@@ -397,11 +493,12 @@ constexpr int CMB_MAX_SLOTS = 256;
 
 struct CmbLayout {
   SelLayout sel;
-  size_t tile, full, empty, xval, ring, total;
+  size_t tile, full, empty, xval, tfull, qtab, ring, total;
 };
 
+// quant: room for QNTB grid tables and their mbarriers.
 __host__ __device__ inline CmbLayout cmb_layout(int I, bool fused, int list_cap, int nslot,
-                                                int slot_bytes) {
+                                                int slot_bytes, bool quant) {
   CmbLayout L;
   size_t o = 0;
   if (fused) {
@@ -412,8 +509,11 @@ __host__ __device__ inline CmbLayout cmb_layout(int I, bool fused, int list_cap,
   L.full = o;  o += 8 * (size_t)nslot;
   L.empty = o; o += 8 * (size_t)nslot;
   L.xval = o;  o += align_up(4 * (size_t)nslot, 16);
+  L.tfull = o; o += quant ? 8 * (size_t)QNTB : 0;
   o = align_up(o, 128);
+  L.qtab = o;  o += quant ? (size_t)QNTB * QTAB_BYTES : 0;
   L.ring = o;  o += (size_t)nslot * slot_bytes;
+  o += quant ? 16 : 0;   // coded walks read one byte past a lane's codes
   L.total = o;
   return L;
 }
@@ -457,6 +557,46 @@ __device__ __forceinline__ void decode_record(const uint8_t* rec, uint16_t xb, f
       acc[t] = fma_f16_f32(*vp, xb, acc[t]);
       ++vp;
     }
+  }
+}
+
+// Coded records (§5, weight-only quantisation): as decode_record / decode_two
+// with b-bit codes in place of the fp16 values; tab is the record's grid
+// table plus lane, so row 32 lane + t's grid is tab[32 t] (conflict-free).
+template <int VB>
+__device__ __forceinline__ void decode_record_q(const uint8_t* rec, uint16_t xb, const uint32_t* tab,
+                                                float (&acc)[32], int lane) {
+  const uint32_t m = reinterpret_cast<const uint32_t*>(rec)[lane];
+  const uint32_t c = __popc(m);
+  const uint32_t incl = warp_inclusive_scan(c, lane);
+  CodeWalk<VB> w;
+  w.init(rec + MASK_BYTES, incl - c);
+#pragma unroll
+  for (int t = 0; t < 32; ++t) {
+    const uint32_t bit = (m >> t) & 1u;
+    acc[t] = q_fma_sel(bit, w.at(), tab[32 * t], xb, acc[t]);
+    w.step(bit);
+  }
+}
+
+template <int VB>
+__device__ __forceinline__ void decode_two_q(const uint8_t* ra, uint16_t xa, const uint32_t* ta,
+                                             const uint8_t* rb, uint16_t xb, const uint32_t* tb,
+                                             float (&acc)[32], int lane) {
+  const uint32_t ma = reinterpret_cast<const uint32_t*>(ra)[lane];
+  const uint32_t mb = reinterpret_cast<const uint32_t*>(rb)[lane];
+  const uint32_t c = (uint32_t)__popc(ma) | ((uint32_t)__popc(mb) << 16);
+  const uint32_t ex = warp_inclusive_scan(c, lane) - c;
+  CodeWalk<VB> wa, wb;
+  wa.init(ra + MASK_BYTES, ex & 0xFFFFu);
+  wb.init(rb + MASK_BYTES, ex >> 16);
+#pragma unroll
+  for (int t = 0; t < 32; ++t) {
+    const uint32_t ba = (ma >> t) & 1u, bb = (mb >> t) & 1u;
+    acc[t] = q_fma_sel(ba, wa.at(), ta[32 * t], xa, acc[t]);
+    acc[t] = q_fma_sel(bb, wb.at(), tb[32 * t], xb, acc[t]);
+    wa.step(ba);
+    wb.step(bb);
   }
 }
 
@@ -504,6 +644,7 @@ struct Resolved {
   const uint8_t* data;   // the product's packed data
   uint32_t o0, o1;       // off[j * S + s], off[j * S + s + 1] (16-byte units)
   uint16_t xb;
+  int g;                 // input-channel group j / 128 (quantised formats)
   bool bad_j;            // channel id out of range
   __device__ __forceinline__ uint32_t bytes() const { return (o1 - o0) * 16u; }
   __device__ __forceinline__ bool bad(int slot_bytes) const {
@@ -527,6 +668,7 @@ __device__ __forceinline__ Resolved resolve_item(const CmbArgs& a, const ItemCur
   }
   r.bad_j = j >= a.I;
   if (r.bad_j) j = 0;   // keep the loads below in bounds; the item is rejected
+  r.g = j / QGROUP;
   const CmbProb& P = a.p[c.p];
   const int64_t ri = (int64_t)j * P.S + c.s;
   r.o0 = __ldg(P.off + ri);
@@ -535,20 +677,25 @@ __device__ __forceinline__ Resolved resolve_item(const CmbArgs& a, const ItemCur
   return r;
 }
 
-template <int MODE>
+template <int MODE, int VB>
 __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArgs a) {
   constexpr bool FUSED = MODE != CMB_LISTED;   // the kernel builds its own kept list
+  constexpr bool QUANT = VB < 16;              // b-bit codes + grid tables (§5)
   extern __shared__ __align__(128) uint8_t sm[];
   __shared__ volatile int abort_flag;
   __shared__ int grid_open;   // 1 once every CTA has zeroed its slice of y
+  __shared__ int cons[CMB_NC];    // QUANT: items each consumer has released
+  __shared__ int tfirst[QNTB];    // QUANT: first item of each table in flight
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nslot = a.nslot, slot_bytes = a.slot_bytes;
-  const CmbLayout L = cmb_layout(a.I, FUSED, a.list_cap, nslot, slot_bytes);
+  const CmbLayout L = cmb_layout(a.I, FUSED, a.list_cap, nslot, slot_bytes, QUANT);
   float* tile = reinterpret_cast<float*>(sm + L.tile);
   uint64_t* full = reinterpret_cast<uint64_t*>(sm + L.full);
   uint64_t* empty = reinterpret_cast<uint64_t*>(sm + L.empty);
   uint32_t* xval = reinterpret_cast<uint32_t*>(sm + L.xval);
   uint8_t* ring = sm + L.ring;
+  uint64_t* tfull = reinterpret_cast<uint64_t*>(sm + L.tfull);
+  uint32_t* qt = reinterpret_cast<uint32_t*>(sm + L.qtab);
   uint16_t* xs = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.xs) : nullptr;
   uint16_t* klist = FUSED ? reinterpret_cast<uint16_t*>(sm + L.sel.klist) : nullptr;
   SelShared* sel = FUSED ? reinterpret_cast<SelShared*>(sm + L.sel.sel) : nullptr;
@@ -563,6 +710,8 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     mbar_init(&full[i], 1);
     mbar_init(&empty[i], 1);
   }
+  if (QUANT && tid < QNTB) mbar_init(&tfull[tid], 1);
+  if (QUANT && tid < CMB_NC) cons[tid] = 0;
   fence_mbar_init();
   if (tid == 0) {
     abort_flag = 0;
@@ -644,13 +793,26 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     ItemCursor cur = cursor_at(u0 + lane);
     SlotCursor sc;
     sc.set(lane, nslot);
-    Resolved q[PQ];
+    Resolved q[PQ] = {};
 #pragma unroll
     for (int d = 0; d < PQ; ++d) {
       if (lane + 32 * d < nv) {
         if (d > 0) cur.advance(a, 32);
         q[d] = resolve_item<FUSED>(a, cur, klist, xs, r0);
       }
+    }
+    // Coded formats: the grid tables of the CTA's run, group gA on, go
+    // through QNTB buffers in order.  Table n (group gA + n) is armed once
+    // every item of a group <= gA + n - QNTB has been released, and an item
+    // is issued only after its table is armed, so a consumer that waits for
+    // table n finds phase n - QNTB of its buffer complete (exact parity).
+    int tarm = 0, last_seq = 0, gA = 0;
+    const uint32_t* qsrc = nullptr;
+    if (QUANT) {
+      const ItemCursor ci = cursor_at(u0);   // a CTA of a coded launch serves one run
+      gA = FUSED ? c0 / QGROUP : __shfl_sync(FULL_MASK, q[0].g, 0);
+      const CmbProb& P = a.p[ci.p];
+      qsrc = P.qtab + ((size_t)ci.s * P.G + gA) * SEG_ROWS;
     }
     // Rounds of 32 items: round R issues items 32 R .. 32 R + 31, lane l the
     // item 32 R + l.  A __syncwarp opens every round, so the rounds run in
@@ -662,31 +824,117 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
         stop = __any_sync(FULL_MASK, stop || abort_flag != 0);
         if (stop) break;
         const int v = R0 + 32 * d + lane;
-        if (v >= nv) continue;
-        const Resolved r = q[d];
-        if (r.bad(slot_bytes)) {
-          atomicOr(&g_status, STATUS_FORMAT);
-          abort_flag = 1;
-          stop = true;
-          continue;
+        if (!QUANT) {
+          if (v >= nv) continue;
+          const Resolved r = q[d];
+          if (r.bad(slot_bytes)) {
+            atomicOr(&g_status, STATUS_FORMAT);
+            abort_flag = 1;
+            stop = true;
+            continue;
+          }
+          if (v + 32 * PQ < nv) {                 // refill: this lane's item v + 32*PQ
+            cur.advance(a, 32);
+            q[d] = resolve_item<FUSED>(a, cur, klist, xs, r0);
+          }
+          // Fill n of a slot waits until fill n - 1 has been consumed.  Fill
+          // n - 1 was issued in an earlier round (nslot >= 32), after fill
+          // n - 2 had been released, so the "empty" phase parity is exact.
+          if (sc.n > 0 && !mbar_wait_bounded(&empty[sc.slot], (uint32_t)((sc.n - 1) & 1), &abort_flag)) {
+            stop = true;
+            continue;
+          }
+          xval[sc.slot] = r.xb;
+          mbar_arrive_expect_tx(&full[sc.slot], r.bytes());
+          bulk_g2s(ring + (size_t)sc.slot * slot_bytes, r.data + (size_t)r.o0 * 16, r.bytes(),
+                   &full[sc.slot], pol);
+          last_v = v;
+          sc.advance(32, nslot);
+        } else {
+          bool pend = v < nv;
+          const Resolved r = q[d];
+          int seq = 0;
+          if (pend) {
+            if (r.bad(slot_bytes)) {
+              atomicOr(&g_status, STATUS_FORMAT);
+              abort_flag = 1;
+              stop = true;
+              pend = false;
+            }
+            if (v + 32 * PQ < nv) {
+              cur.advance(a, 32);
+              q[d] = resolve_item<FUSED>(a, cur, klist, xs, r0);
+            }
+            seq = r.g - gA;
+          }
+          // Groups must not decrease along the items (pending lanes are a
+          // prefix of the warp); a kept list out of group order is rejected.
+          const int prev = __shfl_up_sync(FULL_MASK, seq, 1);
+          if (pend && (seq < 0 || seq < (lane == 0 ? last_seq : prev))) {
+            atomicOr(&g_status, STATUS_FORMAT);
+            abort_flag = 1;
+            stop = true;
+            pend = false;
+          }
+          last_seq = max(last_seq, __reduce_max_sync(FULL_MASK, pend ? seq : 0));
+          while (true) {
+            if (pend && seq < tarm) {   // table armed: issue
+              if (sc.n > 0 &&
+                  !mbar_wait_bounded(&empty[sc.slot], (uint32_t)((sc.n - 1) & 1), &abort_flag)) {
+                stop = true;
+              } else {
+                xval[sc.slot] = (uint32_t)r.xb | ((uint32_t)seq << 16);
+                mbar_arrive_expect_tx(&full[sc.slot], r.bytes());
+                bulk_g2s(ring + (size_t)sc.slot * slot_bytes, r.data + (size_t)r.o0 * 16, r.bytes(),
+                         &full[sc.slot], pol);
+                last_v = v;
+              }
+              pend = false;
+            }
+            const uint32_t pm = __ballot_sync(FULL_MASK, pend);
+            stop = __any_sync(FULL_MASK, stop);
+            if (pm == 0u || stop) break;
+            // Arm table tarm.  Every item of a lower table is issued; the
+            // first item of table >= tarm is the lowest pending lane's.
+            const int b = tarm % QNTB;
+            bool ok = true;
+            if (tarm >= QNTB) {
+              // Its buffer's previous load (table tarm - QNTB) has landed ...
+              if (lane == 0) ok = mbar_wait_bounded(&tfull[b], (uint32_t)((tarm / QNTB - 1) & 1), &abort_flag);
+              ok = __shfl_sync(FULL_MASK, ok, 0);
+              // ... and every item before the first of table tarm - QNTB + 1
+              // is released: lane c checks consumer c's count.
+              const int E = tfirst[(tarm + 1) % QNTB] - 1;
+              const int need = (lane < CMB_NC && E >= lane) ? (E - lane) / CMB_NC + 1 : 0;
+              const int* cw = &cons[lane < CMB_NC ? lane : 0];
+              const uint64_t t0 = globaltimer_ns();
+              while (ok && !__all_sync(FULL_MASK, ld_acquire_cta_shared(cw) >= need)) {
+                const bool late = globaltimer_ns() - t0 > WAIT_LIMIT_NS;
+                if (__any_sync(FULL_MASK, late || abort_flag != 0)) {
+                  if (lane == 0 && late) {
+                    atomicOr(&g_status, STATUS_TIMEOUT);
+                    abort_flag = 1;
+                  }
+                  ok = false;
+                }
+                __nanosleep(32);
+              }
+            }
+            if (!ok) {
+              stop = true;
+              break;
+            }
+            if (lane == 0) {
+              tfirst[b] = R0 + 32 * d + __ffs(pm) - 1;
+              mbar_arrive_expect_tx(&tfull[b], QTAB_BYTES);
+              bulk_g2s(qt + (size_t)b * SEG_ROWS, qsrc + (size_t)tarm * SEG_ROWS, QTAB_BYTES, &tfull[b],
+                       pol);
+            }
+            __syncwarp();
+            ++tarm;
+          }
+          sc.advance(32, nslot);
         }
-        if (v + 32 * PQ < nv) {                 // refill: this lane's item v + 32*PQ
-          cur.advance(a, 32);
-          q[d] = resolve_item<FUSED>(a, cur, klist, xs, r0);
-        }
-        // Fill n of a slot waits until fill n - 1 has been consumed.  Fill
-        // n - 1 was issued in an earlier round (nslot >= 32), after fill
-        // n - 2 had been released, so the "empty" phase parity is exact.
-        if (sc.n > 0 && !mbar_wait_bounded(&empty[sc.slot], (uint32_t)((sc.n - 1) & 1), &abort_flag)) {
-          stop = true;
-          continue;
-        }
-        xval[sc.slot] = r.xb;
-        mbar_arrive_expect_tx(&full[sc.slot], r.bytes());
-        bulk_g2s(ring + (size_t)sc.slot * slot_bytes, r.data + (size_t)r.o0 * 16, r.bytes(),
-                 &full[sc.slot], pol);
-        last_v = v;
-        sc.advance(32, nslot);
       }
       if (stop) break;
     }
@@ -711,6 +959,12 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
         w.set(v, nslot);
         mbar_wait_limited(&full[w.slot], (uint32_t)(w.n & 1));
       }
+    }
+    if (QUANT && lane == 0) {
+      // A table no consumer waited on (a group without kept channels) may
+      // still be landing: wait for the last QNTB before the CTA exits.
+      for (int t = tarm > QNTB ? tarm - QNTB : 0; t < tarm; ++t)
+        mbar_wait_limited(&tfull[t % QNTB], (uint32_t)((t / QNTB) & 1));
     }
   } else {
     // ---------------- consumers ----------------
@@ -751,6 +1005,41 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       return mbar_wait_bounded(&full[q.slot], (uint32_t)(q.n & 1), &abort_flag);
     };
     auto release = [&](const SlotCursor& q) { mbar_arrive(&empty[q.slot]); };
+    // Coded formats: the grid table of an item's group (its table number is
+    // in the slot's xval word), waited for once per table; and the count of
+    // released items, which tells the producer when a table buffer is free.
+    int ncons = 0, cur_seq = -1;
+    const uint32_t* tcur = nullptr;
+    auto table_for = [&](uint32_t seq) -> const uint32_t* {
+      if ((int)seq != cur_seq) {
+        if (!mbar_wait_bounded(&tfull[seq % QNTB], (seq / QNTB) & 1u, &abort_flag)) return nullptr;
+        cur_seq = (int)seq;
+        tcur = qt + (size_t)(seq % QNTB) * SEG_ROWS + lane;
+      }
+      return tcur;
+    };
+    auto released = [&](int n) {   // lane 0, after release()
+      ncons += n;
+      st_release_cta_shared(&cons[c], ncons);
+    };
+    // One coded item, decoded and released before anything else is waited for.
+    auto single_q = [&](const SlotCursor& q, bool& any) {
+      if constexpr (QUANT) {
+        if (!abort_flag && wait_item(q)) {
+          const uint32_t xv = xval[q.slot];
+          const uint32_t* tb = table_for(xv >> 16);
+          if (tb != nullptr) {
+            decode_record_q<VB>(ring + (size_t)q.slot * slot_bytes, (uint16_t)xv, tb, acc, lane);
+            any = true;
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) {
+        release(q);
+        released(1);
+      }
+    };
     // The ring can hold every consumer's partial rows for the final flush.
     const bool scratch_ok = (size_t)nslot * slot_bytes >= (size_t)CMB_NC * SEG_ROWS * sizeof(float);
     uint32_t u = u0;
@@ -770,27 +1059,54 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       if (a.group >= 2) {
         sc2.set(v + CMB_NC, nslot);
         for (; v + CMB_NC < vb; v += 2 * CMB_NC) {   // pairs
-          if (!abort_flag && wait_item(sc) && wait_item(sc2)) {
-            decode_two(ring + (size_t)sc.slot * slot_bytes, (uint16_t)xval[sc.slot],
-                       ring + (size_t)sc2.slot * slot_bytes, (uint16_t)xval[sc2.slot], acc, lane);
-            any = true;
-          }
-          __syncwarp();
-          if (lane == 0) {
-            release(sc);
-            release(sc2);
+          if constexpr (!QUANT) {
+            if (!abort_flag && wait_item(sc) && wait_item(sc2)) {
+              decode_two(ring + (size_t)sc.slot * slot_bytes, (uint16_t)xval[sc.slot],
+                         ring + (size_t)sc2.slot * slot_bytes, (uint16_t)xval[sc2.slot], acc, lane);
+              any = true;
+            }
+            __syncwarp();
+            if (lane == 0) {
+              release(sc);
+              release(sc2);
+            }
+          } else if (FUSED && klist[v] / QGROUP == klist[v + CMB_NC] / QGROUP) {
+            // Same group, same table: holding the first item while waiting
+            // for the second never holds up the arming of a table.
+            if (!abort_flag && wait_item(sc) && wait_item(sc2)) {
+              const uint32_t xa = xval[sc.slot], xb2 = xval[sc2.slot];
+              const uint32_t* tb = table_for(xa >> 16);
+              if (tb != nullptr) {
+                decode_two_q<VB>(ring + (size_t)sc.slot * slot_bytes, (uint16_t)xa, tb,
+                                 ring + (size_t)sc2.slot * slot_bytes, (uint16_t)xb2, tb, acc, lane);
+                any = true;
+              }
+            }
+            __syncwarp();
+            if (lane == 0) {
+              release(sc);
+              release(sc2);
+              released(2);
+            }
+          } else {
+            single_q(sc, any);
+            single_q(sc2, any);
           }
           sc.advance(2 * CMB_NC, nslot);
           sc2.advance(2 * CMB_NC, nslot);
         }
       }
       for (; v < vb; v += CMB_NC) {   // singles
-        if (!abort_flag && wait_item(sc)) {
-          decode_record(ring + (size_t)sc.slot * slot_bytes, (uint16_t)xval[sc.slot], acc, lane);
-          any = true;
+        if constexpr (!QUANT) {
+          if (!abort_flag && wait_item(sc)) {
+            decode_record(ring + (size_t)sc.slot * slot_bytes, (uint16_t)xval[sc.slot], acc, lane);
+            any = true;
+          }
+          __syncwarp();
+          if (lane == 0) release(sc);
+        } else {
+          single_q(sc, any);
         }
-        __syncwarp();
-        if (lane == 0) release(sc);
         sc.advance(CMB_NC, nslot);
       }
       const CmbProb& P = a.p[pc.p];
@@ -885,6 +1201,8 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   const bool thresh = a.thresh != 0;
   const bool fused = thresh || a.kidx == nullptr;
+  const bool quant = a.vbits != 16;
+  if (a.vbits != 16 && a.vbits != 8 && a.vbits != 4) return cudaErrorInvalidValue;
   int64_t total = 0;
   for (int p = 0; p < a.np; ++p) total += (int64_t)a.p[p].S * (thresh ? a.I : a.k);
   if (total <= 0) return cudaSuccess;
@@ -932,8 +1250,8 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
       per_cta = 0;
       for (int q = 0; q < nruns; ++q) per_cta = std::max<int64_t>(per_cta, (a.I + n[q] - 1) / n[q]);
     }
-  } else if (thresh) {
-    return cudaErrorInvalidValue;   // the fused modes need CTAs of their own per run
+  } else if (thresh || quant) {
+    return cudaErrorInvalidValue;   // these launches need CTAs of their own per run
   } else if (fused) {
     return cudaErrorNotSupported;   // the caller selects first and launches with a kept list
   }
@@ -945,18 +1263,28 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   const int slot_bytes = (int)align_up((size_t)std::max(a.slot_bytes, MASK_BYTES + 16), 16);
   if (slot_bytes > MAX_RECORD_BYTES) return cudaErrorInvalidValue;
   const size_t avail = (size_t)dp.smem_optin - 256;   // static shared memory headroom
-  const size_t fixed = cmb_layout(a.I, fused, a.list_cap, 0, slot_bytes).total + 128;
+  const size_t fixed = cmb_layout(a.I, fused, a.list_cap, 0, slot_bytes, quant).total + 128;
   if (fixed >= avail) return cudaErrorInvalidValue;
   int nslot = (int)((avail - fixed) / (slot_bytes + 20));
   nslot = std::min(nslot, CMB_MAX_SLOTS);
   nslot -= nslot % CMB_NC;
   if (nslot < std::max(32, CMB_NC)) return cudaErrorInvalidValue;
-  a.group = nslot >= 2 * CMB_NC ? 2 : 1;   // pairs: waiting for more records costs more than it gains
+  // Pairs (waiting for more records costs more than it gains); coded
+  // formats pair only items of one group, which a consumer can tell ahead
+  // only from the kept list in shared memory (fused modes).
+  a.group = (nslot >= 2 * CMB_NC && (fused || !quant)) ? 2 : 1;
   a.nslot = nslot;
   a.slot_bytes = slot_bytes;
-  const size_t smem = cmb_layout(a.I, fused, a.list_cap, nslot, slot_bytes).total;
-  void (*kern)(const CmbArgs) = thresh ? cmb_spmspv_kernel<CMB_THRESH>
-                                : (fused ? cmb_spmspv_kernel<CMB_TOPK> : cmb_spmspv_kernel<CMB_LISTED>);
+  const size_t smem = cmb_layout(a.I, fused, a.list_cap, nslot, slot_bytes, quant).total;
+  void (*kern)(const CmbArgs) = nullptr;
+  const int mode = thresh ? CMB_THRESH : (fused ? CMB_TOPK : CMB_LISTED);
+#define DUO_CMB_PICK(M, B) \
+  if (mode == M && a.vbits == B) kern = cmb_spmspv_kernel<M, B>;
+  DUO_CMB_PICK(CMB_LISTED, 16) DUO_CMB_PICK(CMB_TOPK, 16) DUO_CMB_PICK(CMB_THRESH, 16)
+  DUO_CMB_PICK(CMB_LISTED, 8) DUO_CMB_PICK(CMB_TOPK, 8) DUO_CMB_PICK(CMB_THRESH, 8)
+  DUO_CMB_PICK(CMB_LISTED, 4) DUO_CMB_PICK(CMB_TOPK, 4) DUO_CMB_PICK(CMB_THRESH, 4)
+#undef DUO_CMB_PICK
+  if (kern == nullptr) return cudaErrorInvalidValue;
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};

@@ -102,7 +102,7 @@ extern "C" int duo_pack_cmb_noalloc(const void* W_fp16_dev, int64_t out, int64_t
   // nothing needs clearing; the previous call's contents are never read.
   rc = map_cuda(duo::launch_pack_count(W, out, in, ldw, (int)S, cnt, st));
   if (rc != DUO_OK) return rc;
-  rc = map_cuda(duo::launch_cmb_offsets(cnt, nrec, off_dev, totals, st));
+  rc = map_cuda(duo::launch_cmb_offsets(cnt, nrec, 16, off_dev, totals, st));
   if (rc != DUO_OK) return rc;
   unsigned long long host_tot[2] = {0, 0};
   rc = map_cuda(cudaMemcpyAsync(host_tot, totals, sizeof(host_tot), cudaMemcpyDeviceToHost, st));
@@ -116,7 +116,7 @@ extern "C" int duo_pack_cmb_noalloc(const void* W_fp16_dev, int64_t out, int64_t
   if (bytes > data_capacity) return DUO_ERANGE;      // *data_bytes tells the size needed
   rc = map_cuda(cudaMemsetAsync(data_dev, 0, (size_t)bytes, st));
   if (rc != DUO_OK) return rc;
-  rc = map_cuda(duo::launch_cmb_scatter(W, out, in, ldw, (int)S, off_dev,
+  rc = map_cuda(duo::launch_cmb_scatter(W, out, in, ldw, (int)S, 16, nullptr, off_dev,
                                         static_cast<uint8_t*>(data_dev), st));
   if (rc != DUO_OK) return rc;
   return map_cuda(cudaStreamSynchronize(st));

@@ -16,8 +16,9 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libduo.so")
 
 DUO_OK, DUO_EINVAL, DUO_ENOMEM, DUO_ECUDA, DUO_ERANGE, DUO_EFORMAT, DUO_ETIMEOUT = 0, -1, -2, -3, -4, -5, -6
-DUO_FMT_IDX16, DUO_FMT_BITMASK = 0, 1
-FORMATS = {"idx16": DUO_FMT_IDX16, "bitmask": DUO_FMT_BITMASK, "cmb": DUO_FMT_BITMASK}
+DUO_FMT_IDX16, DUO_FMT_BITMASK, DUO_FMT_BITMASK_Q8, DUO_FMT_BITMASK_Q4 = 0, 1, 2, 3
+FORMATS = {"idx16": DUO_FMT_IDX16, "bitmask": DUO_FMT_BITMASK, "cmb": DUO_FMT_BITMASK,
+           "bitmask_q8": DUO_FMT_BITMASK_Q8, "bitmask_q4": DUO_FMT_BITMASK_Q4}
 
 _lib = None
 
