@@ -43,3 +43,9 @@ from .duo_oracle import (  # noqa: F401
     ref_unpack_cmb_q,
     required_bytes_q,
 )
+from .calib_oracle import (  # noqa: F401
+    DAMP,
+    sparsify_columns,
+    oracle_calib_precompute,
+    oracle_calib_score,
+)
