@@ -46,6 +46,7 @@ from .duo_oracle import (  # noqa: F401
 from .calib_oracle import (  # noqa: F401
     DAMP,
     sparsify_columns,
+    exact_diag_keys,
     oracle_calib_precompute,
     oracle_calib_score,
 )

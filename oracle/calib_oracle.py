@@ -23,8 +23,10 @@ open; each is listed in DESIGN.md):
     sparsifier does;
   * a channel whose Hessian diagonal is 0 (never kept) gets H_ii = 1;
   * act_order: channels are reordered by the Hessian diagonal, largest first
-    (stable: ties keep the lower index first), and every quantity is in that
-    order; perm[i] is the original channel at position i;
+    (ties keep the lower index first), and every quantity is in that order;
+    perm[i] is the original channel at position i.  The order is decided on
+    the exact diagonal (a sum of squared fp16 values, compared as integers
+    in units of 2^-48), so no rounding can reorder near-equal channels;
   * dampening: H += 0.1 * mean(diag(H)) * I, after the reordering;
   * X_tilde here is the dense input itself (one layer, no earlier pruned
     layer), so dX holds exactly the dropped activations.
@@ -51,6 +53,14 @@ def sparsify_columns(X16, keep: int):
     return Xh
 
 
+def exact_diag_keys(Xh16) -> list[int]:
+    """diag(X_hat X_hat^T) * 2^48 as exact Python integers (every fp16 value
+    is an integer multiple of 2^-24)."""
+    Xh = _as_f16(Xh16)
+    ints = (Xh.astype(np.float64) * 2.0**24).astype(np.int64)
+    return [sum(int(v) * int(v) for v in row) for row in ints]
+
+
 def oracle_calib_precompute(X16, keep: int, damp: float = DAMP, act_order: bool = True):
     """The precompute of Algorithm 1 (readings in the module docstring).
 
@@ -62,11 +72,12 @@ def oracle_calib_precompute(X16, keep: int, damp: float = DAMP, act_order: bool 
     Xh = Xh16.astype(np.float64)
     Xt = X.astype(np.float64)
     H = Xh @ Xh.T
-    d = np.diag(H).copy()
-    dead = d == 0
+    key = exact_diag_keys(Xh16)
+    dead = np.array([kk == 0 for kk in key])
     H[dead, dead] = 1.0
+    key = [kk if kk != 0 else 1 << 48 for kk in key]   # H_ii = 1 for a dead channel
     if act_order:
-        perm = np.lexsort((np.arange(k), -np.diag(H)))   # largest diagonal first, ties by index
+        perm = np.array(sorted(range(k), key=lambda i: (-key[i], i)), dtype=np.int64)
     else:
         perm = np.arange(k)
     H = H[np.ix_(perm, perm)]
