@@ -57,8 +57,13 @@ def exact_diag_keys(Xh16) -> list[int]:
     """diag(X_hat X_hat^T) * 2^48 as exact Python integers (every fp16 value
     is an integer multiple of 2^-24)."""
     Xh = _as_f16(Xh16)
-    ints = (Xh.astype(np.float64) * 2.0**24).astype(np.int64)
-    return [sum(int(v) * int(v) for v in row) for row in ints]
+    v = np.abs((Xh.astype(np.float64) * 2.0**24).astype(np.int64))   # < 2^40
+    hi, lo = v >> 20, v & ((1 << 20) - 1)                            # v = hi 2^20 + lo
+    # v^2 = hi^2 2^40 + 2 hi lo 2^20 + lo^2; each column sum stays below 2^63
+    shh = (hi * hi).sum(axis=1)
+    shl = (hi * lo).sum(axis=1)
+    sll = (lo * lo).sum(axis=1)
+    return [(int(a) << 40) + (int(b) << 21) + int(c) for a, b, c in zip(shh, shl, sll)]
 
 
 def oracle_calib_precompute(X16, keep: int, damp: float = DAMP, act_order: bool = True):

@@ -17,9 +17,14 @@ constexpr int MAXP = 4;                  // products per multi launch
 constexpr uint64_t WAIT_LIMIT_NS = 1000000000ull;  // 1 s per bounded wait
 
 // Device status word (bit 0: a bounded wait ran out; bit 1: a record size or
-// channel id outside the format's bounds).  Defined here because this header
-// is included by exactly one translation unit (kernels.cu).
+// channel id outside the format's bounds), read by duo_device_status.  The
+// translation unit that owns it (kernels.cu) defines DUO_STATUS_OWNER; any
+// other unit including this header gets a private copy nobody reads.
+#ifdef DUO_STATUS_OWNER
 __device__ unsigned int g_status = 0u;
+#else
+static __device__ unsigned int g_status = 0u;
+#endif
 constexpr unsigned int STATUS_TIMEOUT = 1u;
 constexpr unsigned int STATUS_FORMAT = 2u;
 

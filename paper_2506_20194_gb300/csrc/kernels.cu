@@ -6,6 +6,7 @@
 #include <algorithm>
 #include <cstdio>
 
+#define DUO_STATUS_OWNER
 #include "duo_device.cuh"
 #include "duo_launch.h"
 

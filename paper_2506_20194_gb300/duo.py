@@ -60,11 +60,19 @@ def load_library(path: str | None = None):
     lib.duo_packed_export.argtypes = [vp, i32, vp, i64]
     lib.duo_pack_cmb_noalloc.argtypes = [vp, i64, i64, i64, vp, vp, i64, ctypes.POINTER(i64), vp]
     lib.duo_device_status.argtypes = [vp]
+    lib.duo_calib_create.argtypes = [i64, i64, vp, ctypes.POINTER(vp)]
+    lib.duo_calib_precompute.argtypes = [vp, vp, i64, ctypes.c_float, i32, vp]
+    lib.duo_calib_status.argtypes = [vp, vp]
+    lib.duo_calib_export.argtypes = [vp, i32, vp, i64, vp]
+    lib.duo_calib_score.argtypes = [vp, vp, i64, i64, vp, vp]
+    lib.duo_calib_free.argtypes = [vp]
     lib.duo_strerror.argtypes = [i32]
     lib.duo_strerror.restype = ctypes.c_char_p
     for name in ("duo_pack", "duo_sparsify", "duo_spmspv", "duo_spmspv_multi", "duo_free",
                  "duo_packed_query", "duo_packed_export", "duo_device_status", "duo_abi_version",
-                 "duo_pack_cmb_noalloc", "duo_sparsify_threshold", "duo_spmspv_threshold"):
+                 "duo_pack_cmb_noalloc", "duo_sparsify_threshold", "duo_spmspv_threshold",
+                 "duo_calib_create", "duo_calib_precompute", "duo_calib_status", "duo_calib_export",
+                 "duo_calib_score", "duo_calib_free"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -272,3 +280,61 @@ def duo_pack_cmb_noalloc(W: torch.Tensor, off: torch.Tensor | None = None,
     _check(lib.duo_pack_cmb_noalloc(W.data_ptr(), O, I, W.stride(0), off.data_ptr(), data.data_ptr(),
                                     data.numel(), ctypes.byref(nb), st), "duo_pack_cmb_noalloc")
     return off, data, nb.value
+
+
+_CALIB_BUFS = {"perm": (0, torch.int32, 1), "H": (1, torch.float32, 2), "L": (2, torch.float32, 2),
+               "Q": (3, torch.float32, 2), "U": (4, torch.float32, 2), "D": (5, torch.float32, 2),
+               "a": (6, torch.float32, 1), "b": (7, torch.float32, 1), "c": (8, torch.float32, 1),
+               "col": (9, torch.float32, 1)}
+
+
+class Calib:
+    """Context of the calibration precompute (§4.3, Algorithm 1) for k
+    channels and m tokens; see include/duo_calib.h."""
+
+    def __init__(self, k: int, m: int, stream=None):
+        h = ctypes.c_void_p()
+        _check(load_library().duo_calib_create(int(k), int(m), _stream_ptr(stream), ctypes.byref(h)),
+               "duo_calib_create")
+        self._h, self.k, self.m = h.value, int(k), int(m)
+
+    def precompute(self, X: torch.Tensor, keep: int, damp: float = 0.1, act_order: bool = True,
+                   stream=None):
+        """X: m x k fp16 CUDA tensor, one row per token (the paper's X is k x m)."""
+        if X.dtype != torch.float16 or tuple(X.shape) != (self.m, self.k) or not X.is_contiguous():
+            raise DuoError(DUO_EINVAL, "precompute needs a contiguous m x k fp16 tensor")
+        _check(load_library().duo_calib_precompute(self._h, X.data_ptr(), int(keep), float(damp),
+                                                   1 if act_order else 0, _stream_ptr(stream)),
+               "duo_calib_precompute")
+
+    def status(self, stream=None) -> int:
+        return load_library().duo_calib_status(self._h, _stream_ptr(stream))
+
+    def get(self, name: str, stream=None) -> torch.Tensor:
+        which, dt, nd = _CALIB_BUFS[name]
+        shape = (self.k, self.k) if nd == 2 else (self.k,)
+        out = torch.empty(shape, dtype=dt, device="cuda")
+        _check(load_library().duo_calib_export(self._h, which, out.data_ptr(), out.numel() * 4,
+                                               _stream_ptr(stream)), "duo_calib_export")
+        return out
+
+    def score(self, W: torch.Tensor, S: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+        """S = W^2 (1 / L_pp^2 + a - b + 2 c), columns in the processing order."""
+        if W.dtype != torch.float16 or W.dim() != 2 or W.shape[1] != self.k or W.stride(1) != 1:
+            raise DuoError(DUO_EINVAL, "score needs an n x k fp16 tensor with unit column stride")
+        if S is None:
+            S = torch.empty(W.shape[0], self.k, dtype=torch.float32, device=W.device)
+        _check(load_library().duo_calib_score(self._h, W.data_ptr(), W.shape[0], W.stride(0),
+                                              S.data_ptr(), _stream_ptr(stream)), "duo_calib_score")
+        return S
+
+    def free(self):
+        if self._h:
+            h, self._h = self._h, None
+            _check(load_library().duo_calib_free(h), "duo_calib_free")
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass

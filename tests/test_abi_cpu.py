@@ -1,5 +1,5 @@
 """C ABI checks that need no GPU: the library builds and loads, exports every
-function include/duo.h declares, and rejects invalid arguments on the host
+function include/*.h declares, and rejects invalid arguments on the host
 before any device work (no pointer below is ever dereferenced)."""
 import ctypes
 import os
@@ -8,7 +8,8 @@ import re
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-HEADER = os.path.join(ROOT, "include", "duo.h")
+HEADERS = [os.path.join(ROOT, "include", f) for f in sorted(os.listdir(os.path.join(ROOT, "include")))
+           if f.endswith(".h")]
 
 
 @pytest.fixture(scope="module")
@@ -20,7 +21,7 @@ def lib():
 
 
 def _declared_functions():
-    txt = open(HEADER).read()
+    txt = "\n".join(open(h).read() for h in HEADERS)
     txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
     return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(duo_\w+)\s*\(", txt, flags=re.M)))
 
@@ -29,13 +30,15 @@ def test_header_declares_the_boundary():
     names = _declared_functions()
     for n in ("duo_pack", "duo_sparsify", "duo_spmspv", "duo_spmspv_multi", "duo_free",
               "duo_strerror", "duo_packed_query", "duo_packed_export", "duo_device_status",
-              "duo_abi_version"):
+              "duo_abi_version", "duo_sparsify_threshold", "duo_spmspv_threshold",
+              "duo_calib_create", "duo_calib_precompute", "duo_calib_status", "duo_calib_query",
+              "duo_calib_export", "duo_calib_score", "duo_calib_free"):
         assert n in names
 
 
 def test_library_exports_every_declared_symbol(lib):
     for n in _declared_functions():
-        assert hasattr(lib, n), f"{n} declared in duo.h but not exported"
+        assert hasattr(lib, n), f"{n} declared in include/ but not exported"
 
 
 def test_abi_version_and_strerror(lib):
@@ -121,3 +124,28 @@ def test_binding_fails_loudly_without_library(tmp_path):
             duo.load_library(str(tmp_path / "missing.so"))
     finally:
         duo._lib = saved
+
+
+def test_calib_argument_validation(lib):
+    EINVAL = -1
+    vp, i64 = ctypes.c_void_p, ctypes.c_int64
+    lib.duo_calib_create.argtypes = [i64, i64, vp, ctypes.POINTER(vp)]
+    lib.duo_calib_precompute.argtypes = [vp, vp, i64, ctypes.c_float, ctypes.c_int, vp]
+    lib.duo_calib_score.argtypes = [vp, vp, i64, i64, vp, vp]
+    lib.duo_calib_free.argtypes = [vp]
+    lib.duo_calib_status.argtypes = [vp, vp]
+    lib.duo_calib_export.argtypes = [vp, ctypes.c_int, vp, i64, vp]
+    h = ctypes.c_void_p()
+    assert lib.duo_calib_create(0, 8, None, ctypes.byref(h)) == EINVAL
+    assert lib.duo_calib_create(8, 0, None, ctypes.byref(h)) == EINVAL
+    assert lib.duo_calib_create(40000, 8, None, ctypes.byref(h)) == EINVAL
+    assert lib.duo_calib_create(8, 8, None, None) == EINVAL
+    assert h.value is None
+    # an unknown handle is rejected before it is dereferenced
+    assert lib.duo_calib_precompute(FAKE, FAKE, 1, 0.1, 1, None) == EINVAL
+    assert lib.duo_calib_precompute(None, FAKE, 1, 0.1, 1, None) == EINVAL
+    assert lib.duo_calib_score(FAKE, FAKE, 4, 8, FAKE, None) == EINVAL
+    assert lib.duo_calib_status(FAKE, None) == EINVAL
+    assert lib.duo_calib_export(FAKE, 0, FAKE, 32, None) == EINVAL
+    assert lib.duo_calib_free(FAKE) == EINVAL
+    assert lib.duo_calib_free(None) == 0

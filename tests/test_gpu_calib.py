@@ -1,0 +1,101 @@
+"""GPU parity of the calibration precompute (§4.3, Algorithm 1) through the
+C ABI (include/duo_calib.h) against the fp64 CPU oracle.
+
+Bars: the act_order permutation is bit-exact (both sides decide it on the
+exact Hessian diagonal).  The fp32 quantities are compared normwise:
+max |x_gpu - x_ref| <= tol * max |x_ref| per quantity, with tol = 1e-5 for H
+and a (fp16 products, fp32 sums) and 2e-3 for what goes through the fp32
+factorisation (L, Q, U, D, b, c, col, S).  The factorisation's error grows
+like k u kappa(H) (u = 2^-24); with the 0.1 dampening kappa(H) stays small
+for these inputs, and 2e-3 leaves a wide margin over the errors observed.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+
+pytestmark = pytest.mark.gpu
+
+TOL_EXACTISH = 1e-5
+TOL_FACTOR = 2e-3
+
+
+@pytest.fixture(scope="module")
+def duo():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2506_20194_gb300 import duo as d
+    d.load_library()
+    return d
+
+
+def _inputs(k, m, seed, dead=False):
+    rng = np.random.default_rng(seed)
+    X = rng.laplace(0, 1, size=(k, m)).astype(np.float16)    # the paper's k x m
+    if dead:
+        X[1] = np.float16(1e-3)       # never among the largest: H_ii = 0
+    return X
+
+
+def _close(name, got, want, tol):
+    got = np.asarray(got, dtype=np.float64)
+    scale = max(np.abs(want).max(), 1e-30)
+    err = np.abs(got - want).max()
+    assert err <= tol * scale, f"{name}: max err {err:.3e} vs {tol:.0e} * {scale:.3e}"
+
+
+def _check(duo, k, m, keep, act_order, seed, dead=False):
+    X = _inputs(k, m, seed, dead)
+    pre = orc.oracle_calib_precompute(X, keep, act_order=act_order)
+    c = duo.Calib(k, m)
+    c.precompute(torch.from_numpy(np.ascontiguousarray(X.T)).cuda(), keep, 0.1, act_order)
+    assert c.status() == 0
+    assert c.get("perm").cpu().numpy().tolist() == pre["perm"].tolist()
+    _close("H", c.get("H").cpu().numpy(), pre["H"], TOL_EXACTISH)
+    _close("a", c.get("a").cpu().numpy(), pre["a"], TOL_EXACTISH)
+    for name in ("L", "Q", "U", "D"):
+        _close(name, c.get(name).cpu().numpy(), pre[name], TOL_FACTOR)
+    for name in ("b", "c"):
+        _close(name, c.get(name).cpu().numpy(), pre[name], TOL_FACTOR)
+    col_ref = 1.0 / np.diag(pre["L"]) ** 2 + pre["a"] - pre["b"] + 2 * pre["c"]
+    _close("col", c.get("col").cpu().numpy(), col_ref, TOL_FACTOR)
+    rng = np.random.default_rng(seed + 1)
+    W = (rng.standard_normal((37, k)) * 0.02).astype(np.float16)
+    S = c.score(torch.from_numpy(W).cuda()).cpu().numpy()
+    _close("S", S, orc.oracle_calib_score(W, pre), TOL_FACTOR)
+    c.free()
+
+
+@pytest.mark.parametrize("k,m,keep,act_order", [(64, 128, 32, True), (64, 128, 32, False),
+                                                 (200, 300, 100, True), (256, 512, 77, True),
+                                                 (256, 512, 256, True), (128, 64, 1, True)])
+def test_precompute_matches_oracle(duo, k, m, keep, act_order):
+    _check(duo, k, m, keep, act_order, seed=k * 7 + m + keep)
+
+
+def test_precompute_dead_channel(duo):
+    _check(duo, 96, 200, 48, True, seed=5, dead=True)
+
+
+def test_precompute_full_size_layer(duo):
+    """The bench's shape: 4096 channels, 2048 tokens, half the channels kept."""
+    _check(duo, 4096, 2048, 2048, True, seed=11)
+
+
+def test_context_reuse_and_errors(duo):
+    k, m = 64, 96
+    c = duo.Calib(k, m)
+    X = torch.from_numpy(np.ascontiguousarray(_inputs(k, m, 3).T)).cuda()
+    for keep in (16, 48):
+        c.precompute(X, keep)
+        assert c.status() == 0
+    with pytest.raises(duo.DuoError):
+        c.precompute(X, k + 1)
+    with pytest.raises(duo.DuoError):
+        c.precompute(X, 8, damp=-1.0)
+    c.free()
+    with pytest.raises(duo.DuoError):
+        c.precompute(X, 8)
