@@ -251,9 +251,16 @@ def max_over_ranks(v, world):
     if world == 1:
         return v
     import torch.distributed as dist
-    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job_gbs(bytes_per_step, steps, world, seconds):
+    """Whole-job throughput of N replicas: every rank moves bytes_per_step
+    per step, the time is the slowest rank's."""
+    return bytes_per_step * steps * world / seconds / 1e9
 
 
 # --------------------------------------------------------- CPU oracle arm --
@@ -379,7 +386,7 @@ def run_ours(args):
     t = max_over_ranks(t, world)
     assert duo.duo_device_status() == duo.DUO_OK
     us_layer = t / steps_timed * 1e6
-    value = breq_mean * steps_timed * world / t / 1e9
+    value = whole_job_gbs(breq_mean, steps_timed, world, t)
 
     # Average launch duration of the fused kernel per stage: a graph of that
     # stage's launch for every layer, timed with CUDA events on the stream.
@@ -425,6 +432,7 @@ def run_ours(args):
 
     thresh = run_threshold_path(duo, shape, layers, args.px, reps, peak)
     quant = {f"int{b}": run_quant_path(duo, shape, layers, args.px, reps, peak, b) for b in (8, 4)}
+    calib = run_calib(duo, reps)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -450,6 +458,7 @@ def run_ours(args):
             "sweep_px": sweep,
             "threshold_path": thresh,
             "quantised_values": quant,
+            "calibration_precompute": calib,
         }
         print(json.dumps(line), flush=True)
     for lay in layers:
@@ -548,6 +557,45 @@ def run_quant_path(duo, shape, layers, px, reps, peak, bits):
     return {"us_per_layer": us, "GB/s": gbs, "frac_of_peak": gbs / peak, "required_MB": breq / 1e6,
             "packed_MB_per_layer": packed / 1e6, "bits": bits, "group": 128,
             "grid": "asymmetric min-max per (row, 128-channel group), fp16 scale, RTN"}
+
+
+def run_calib(duo, reps):
+    """DuoGPT's calibration precompute (§4.3, Algorithm 1) for one
+    4096-channel layer from 2048 calibration tokens with half the channels
+    kept per token (the setting of the paper's efficiency measurement):
+    duo_calib_precompute (sparse input, H, act_order, dampening, inverse
+    Cholesky, Q, U, a, b, c, D) and the score S of a 4096 x 4096 weight.
+    Synthetic inputs: Laplace(0, 1) activations, N(0, 0.02) weights."""
+    k, m = 4096, 2048
+    keep = k // 2
+    g = torch.Generator(device="cuda").manual_seed(2506)
+    u = torch.rand(m, k, generator=g, device="cuda", dtype=torch.float32) - 0.5
+    X = (-torch.sign(u) * torch.log1p(-2 * u.abs())).to(torch.float16)
+    W = (torch.randn(k, k, generator=g, device="cuda") * 0.02).to(torch.float16)
+    c = duo.Calib(k, m)
+    S = torch.empty(k, k, dtype=torch.float32, device="cuda")
+    for _ in range(3):
+        c.precompute(X, keep)
+        c.score(W, S)
+    status = c.status()
+    r = max(3, min(reps // 20, 20))
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    ev[0].record()
+    for _ in range(r):
+        c.precompute(X, keep)
+    ev[1].record()
+    for _ in range(r):
+        c.score(W, S)
+    ev[2].record()
+    torch.cuda.synchronize()
+    pre_ms = ev[0].elapsed_time(ev[1]) / r
+    score_ms = ev[1].elapsed_time(ev[2]) / r
+    gemm_flop = 4.0 * k * k * m + 4.0 * k ** 3     # H, dX X_hat^T, Q, D as issued
+    c.free()
+    return {"k": k, "m": m, "keep": keep, "status": status, "precompute_ms": pre_ms,
+            "score_ms": score_ms, "gemm_GFLOP": gemm_flop / 1e9,
+            "gemm_TFLOP/s_over_precompute": gemm_flop / (pre_ms * 1e-3) / 1e12,
+            "paper_context": "about 1 ms for a, b, c and S of a 4096 x 4096 layer, m = 2048, A100 (App. C)"}
 
 
 def run_e2e(duo, shape, layers, args, breq_mean):

@@ -1,0 +1,50 @@
+"""The N > 1 path of bench.py (replicas, no data-path collective) on CPU:
+two gloo ranks on 127.0.0.1 go through the same setup, barrier and
+max-over-ranks timing the GPU run uses, and the whole-job value counts
+every rank's bytes over the slowest rank's time."""
+import os
+import socket
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, out):
+    os.environ.update(RANK=str(rank), WORLD_SIZE=str(world), LOCAL_RANK=str(rank),
+                      MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    sys.path.insert(0, ROOT)
+    import bench
+    import torch.distributed as dist
+    w, r, local = bench.dist_setup(None)
+    assert (w, r, local) == (world, rank, rank)
+    assert dist.get_backend() == "gloo"
+    bench.barrier(w)
+    t = bench.max_over_ranks(1.0 + rank, w)          # rank 1 is the slower one
+    out.put((rank, t, bench.whole_job_gbs(1e9, 10, w, t)))
+    bench.barrier(w)
+    dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_take_the_slowest_time():
+    ctx = mp.get_context("spawn")
+    out = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=120)
+        assert p.exitcode == 0
+    res = sorted(out.get(timeout=10) for _ in range(2))
+    for rank, t, gbs in res:
+        assert t == 2.0                                  # max over ranks
+        assert gbs == pytest.approx(1e9 * 10 * 2 / 2.0 / 1e9)
