@@ -36,8 +36,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch of
 # the fused kernel from one ncu capture, valid only for the kernel source it
 # was taken on (sha256 of kernels.cu + duo_device.cuh, first 16 hex digits).
-TRAFFIC = {"sha": "05dc308352cf79df",
-           "per_launch_bytes": [29106176.0, 9754624.0, 51912448.0, 26100736.0]}
+TRAFFIC = {"sha": "3acf777159afa7db",
+           "per_launch_bytes": [29105664.0, 9753088.0, 51889152.0, 26097920.0]}
 
 
 def parse():
@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--profile", action="store_true",
                     help="small case for ncu: 2 layers, a few direct (ungraphed) layer steps")
+    ap.add_argument("--profile-calib", action="store_true",
+                    help="small case for ncu: `--steps` calibration precomputes of a 4096-channel layer")
     ap.add_argument("--stack", default=None,
                     choices=("llama2-7b-layer", "llama3-8b-stack", "llama2-13b-stack", "llama2-70b-stack"),
                     help="per-token time over every layer of a stack workload (one CUDA graph per token)")
@@ -672,6 +674,26 @@ def run_profile(args):
     print("profile workload done", flush=True)
 
 
+def run_profile_calib(args):
+    """Calibration precompute for profiler captures: one 4096-channel layer
+    from 2048 tokens, one warm-up and `--steps` precomputes, no graphs."""
+    torch.cuda.set_device(0)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2506_20194_gb300 import duo
+    duo.load_library()
+    k, m = 4096, 2048
+    g = torch.Generator(device="cuda").manual_seed(2506)
+    u = torch.rand(m, k, generator=g, device="cuda", dtype=torch.float32) - 0.5
+    X = (-torch.sign(u) * torch.log1p(-2 * u.abs())).to(torch.float16)
+    c = duo.Calib(k, m)
+    for _ in range(1 + args.steps):
+        c.precompute(X, k // 2)
+    assert c.status() == duo.DUO_OK
+    c.free()
+    print("profile workload done", flush=True)
+
+
 def run_stack(args):
     """Per-token time of a whole stack: every layer's four launches (q/k/v,
     o, gate/up, down) in one CUDA graph, each layer with its own packed
@@ -739,6 +761,8 @@ def main():
     args = parse()
     if args.profile:
         run_profile(args)
+    elif args.profile_calib:
+        run_profile_calib(args)
     elif args.stack is not None:
         run_stack(args)
     elif args.impl == "reference":
