@@ -49,4 +49,6 @@ from .calib_oracle import (  # noqa: F401
     exact_diag_keys,
     oracle_calib_precompute,
     oracle_calib_score,
+    oracle_calib_prune,
+    oracle_calib_prune_blocked,
 )

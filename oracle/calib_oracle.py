@@ -109,3 +109,88 @@ def oracle_calib_score(W16, pre) -> np.ndarray:
     L = pre["L"]
     col = 1.0 / np.diag(L) ** 2 + pre["a"] - pre["b"] + 2.0 * pre["c"]
     return W * W * col[None, :]
+
+
+def oracle_calib_prune(W16, pre, pw_pct: int, block: int = 128):
+    """Algorithm 1's column sweep (§4.3) after the precompute `pre`, written
+    unblocked: columns in the processing order; at the first column of every
+    block of `block` columns, the scores of the block's current weights
+    S = W^2 (1 / L_pp^2 + a - b + 2 c) decide its mask: the
+    floor(n * B_j * pw_pct / 100) weights of the block with the lowest scores
+    are pruned (equal scores: the lower flat index r * B_j + c first); then
+    for each column j, P_j = W_j (.) M_j, E_j = (W_j - P_j) / L_jj, and every
+    later column q gets W_q -= E_j L_qj - W_j D_jq (W_j as it is at step j),
+    after which W_j = P_j.  This equals the blocked form with lazy batch
+    updates when the trailing columns see the same W_j (the reading taken).
+
+    Returns (W_pruned fp64 n x k in the ORIGINAL channel order, keep mask
+    bool n x k in the original order)."""
+    W = _as_f16(W16).astype(np.float64)
+    n, k = W.shape
+    perm = pre["perm"]
+    L, D = pre["L"], pre["D"]
+    col = 1.0 / np.diag(L) ** 2 + pre["a"] - pre["b"] + 2.0 * pre["c"]
+    Wp = W[:, perm].copy()
+    keep = np.ones((n, k), dtype=bool)
+    for i in range(0, k, block):
+        bj = min(block, k - i)
+        S = Wp[:, i:i + bj] ** 2 * col[None, i:i + bj]
+        cnt = (n * bj * pw_pct) // 100
+        flat = S.reshape(-1)
+        order = np.lexsort((np.arange(flat.size), flat))     # score, then flat index
+        m = np.ones(flat.size, dtype=bool)
+        m[order[:cnt]] = False
+        keep[:, i:i + bj] = m.reshape(n, bj)
+        for j in range(i, i + bj):
+            wj = Wp[:, j].copy()
+            pj = np.where(keep[:, j], wj, 0.0)
+            E = (wj - pj) / L[j, j]
+            if j + 1 < k:
+                Wp[:, j + 1:] -= np.outer(E, L[j + 1:, j]) - np.outer(wj, D[j, j + 1:])
+            Wp[:, j] = pj
+    out = np.zeros_like(Wp)
+    out[:, perm] = Wp
+    mask = np.zeros_like(keep)
+    mask[:, perm] = keep
+    return out, mask
+
+
+def oracle_calib_prune_blocked(W16, pre, pw_pct: int, block: int = 128):
+    """The same sweep in Algorithm 1's blocked form: within a block the
+    updates reach only the block's columns; at the block's end the trailing
+    columns get W_T -= E L_T,blk^T - W_pre D_blk,T in one product (lazy
+    batch), W_pre holding each block column as it was at its step."""
+    W = _as_f16(W16).astype(np.float64)
+    n, k = W.shape
+    perm = pre["perm"]
+    L, D = pre["L"], pre["D"]
+    col = 1.0 / np.diag(L) ** 2 + pre["a"] - pre["b"] + 2.0 * pre["c"]
+    Wp = W[:, perm].copy()
+    keep = np.ones((n, k), dtype=bool)
+    for i in range(0, k, block):
+        bj = min(block, k - i)
+        S = Wp[:, i:i + bj] ** 2 * col[None, i:i + bj]
+        cnt = (n * bj * pw_pct) // 100
+        flat = S.reshape(-1)
+        order = np.lexsort((np.arange(flat.size), flat))
+        m = np.ones(flat.size, dtype=bool)
+        m[order[:cnt]] = False
+        keep[:, i:i + bj] = m.reshape(n, bj)
+        E = np.zeros((n, bj))
+        Wpre = np.zeros((n, bj))
+        for jj in range(bj):
+            j = i + jj
+            Wpre[:, jj] = Wp[:, j]
+            pj = np.where(keep[:, j], Wp[:, j], 0.0)
+            E[:, jj] = (Wp[:, j] - pj) / L[j, j]
+            if jj + 1 < bj:
+                Wp[:, j + 1:i + bj] -= np.outer(E[:, jj], L[j + 1:i + bj, j]) - np.outer(Wpre[:, jj], D[j, j + 1:i + bj])
+            Wp[:, j] = pj
+        if i + bj < k:
+            T = slice(i + bj, k)
+            Wp[:, T] -= E @ L[T, i:i + bj].T - Wpre @ D[i:i + bj, T]
+    out = np.zeros_like(Wp)
+    out[:, perm] = Wp
+    mask = np.zeros_like(keep)
+    mask[:, perm] = keep
+    return out, mask

@@ -167,3 +167,65 @@ def test_invariants_of_L_perm_and_sparse_input():
     # a = per-channel energy of the dropped activations
     np.testing.assert_allclose(pre["a"], np.sum(pre["dX"] ** 2, axis=1))
     assert np.all(pre["dX"] * pre["Xh"] == 0)   # each entry is kept or dropped, not both
+
+
+# ------------------------------------------------------------ column sweep ----
+
+def test_sweep_golden_cases():
+    g = _parse_golden()
+    pre = orc.oracle_calib_precompute(g["X"].astype(np.float16), 1)
+    for wn, rn in (("Wsweep1", "result1"), ("Wsweep2", "result2")):
+        W = g[wn].astype(np.float16)[None, :]
+        Wf, keep = orc.oracle_calib_prune(W, pre, 50, block=2)
+        np.testing.assert_allclose(Wf[0], g[rn], rtol=1e-12, atol=1e-15)
+        assert keep[0].tolist() == [bool(v != 0) for v in g[rn]]
+
+
+def _sweep_inputs(seed, n, k, m, keep):
+    rng = np.random.default_rng(seed)
+    X = rng.laplace(0, 1, size=(k, m)).astype(np.float16)
+    W = (rng.standard_normal((n, k)) * 0.05).astype(np.float16)
+    return X, W, orc.oracle_calib_precompute(X, keep)
+
+
+@pytest.mark.parametrize("n,k,m,keep,block,pw", [(8, 24, 40, 12, 8, 50), (5, 30, 50, 10, 7, 60),
+                                                 (6, 16, 30, 16, 16, 25)])
+def test_sweep_blocked_equals_unblocked(n, k, m, keep, block, pw):
+    """Algorithm 1's blocked form (lazy batch updates) against the column by
+    column form: the same masks and, up to rounding, the same weights."""
+    X, W, pre = _sweep_inputs(n * k + m, n, k, m, keep)
+    Wu, mu = orc.oracle_calib_prune(W, pre, pw, block)
+    Wb, mb = orc.oracle_calib_prune_blocked(W, pre, pw, block)
+    assert np.array_equal(mu, mb)
+    np.testing.assert_allclose(Wb, Wu, rtol=1e-10, atol=1e-12 * np.abs(Wu).max())
+
+
+def test_sweep_masks_and_pruned_zeros():
+    n, k, m, block, pw = 10, 40, 60, 16, 50
+    X, W, pre = _sweep_inputs(9, n, k, m, 20)
+    Wf, keep = orc.oracle_calib_prune(W, pre, pw, block)
+    assert np.all(Wf[~keep] == 0)
+    kp = keep[:, pre["perm"]]                       # processing order
+    for i in range(0, k, block):
+        bj = min(block, k - i)
+        assert (~kp[:, i:i + bj]).sum() == (n * bj * pw) // 100
+    # the first block's decision is on the original weights: its pruned
+    # scores are all at or below its kept ones
+    col = 1.0 / np.diag(pre["L"]) ** 2 + pre["a"] - pre["b"] + 2 * pre["c"]
+    S0 = W.astype(np.float64)[:, pre["perm"][:block]] ** 2 * col[:block]
+    assert S0[~kp[:, :block]].max() <= S0[kp[:, :block]].min()
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_sweep_compensation_lowers_the_calibration_loss(seed):
+    """The point of the sweep (§4.2): with the same mask, the compensated
+    weights reproduce the dense output W X_tilde from the sparse input better
+    than the masked weights alone."""
+    n, k, m = 12, 48, 200
+    X, W, pre = _sweep_inputs(100 + seed, n, k, m, 24)
+    Wf, keep = orc.oracle_calib_prune(W, pre, 50, 16)
+    Xh = orc.sparsify_columns(X, 24).astype(np.float64)
+    target = W.astype(np.float64) @ X.astype(np.float64)
+    loss_comp = np.linalg.norm(Wf @ Xh - target)
+    loss_mask = np.linalg.norm(np.where(keep, W.astype(np.float64), 0.0) @ Xh - target)
+    assert loss_comp < loss_mask
