@@ -111,6 +111,31 @@ int duo_calib_export(const duo_calib* h, int which, void* dst_dev, int64_t bytes
 int duo_calib_score(const duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw,
                     float* S_dev, void* stream);
 
+/*
+ * duo_calib_prune -- Algorithm 1's column sweep for the last precompute: in
+ * the processing order, blocks of `block` columns; at each block's start the
+ * scores S = W^2 (1 / L_pp^2 + a - b + 2 c) of its current weights choose
+ * the floor(n * B_j * pw_pct / 100) weights to prune (lowest scores; equal
+ * scores: lower flat index r * B_j + c first); then column by column
+ * P_j = W_j M_j, E_j = (W_j - P_j) / L_jj and later columns q get
+ * W_q -= E_j L_qj - W_j D_jq (within the block at once, for the columns
+ * after the block in one lazy product that uses each W_j as it was at its
+ * step); finally W_j = P_j.  Asynchronous; the context keeps scratch of
+ * about n k (4 + 1) bytes, grown when a call needs more rows (growing waits
+ * for the stream).
+ *   W_fp16_dev : device fp16, n x k row-major (leading dimension ldw), the
+ *                dense weight in the ORIGINAL channel order.
+ *   pw_pct     : weight sparsity in percent, 0..100.   block : 1..128 (the
+ *                paper uses 128).
+ *   Wout_dev   : device fp32, n x k row-major: the pruned and compensated
+ *                weight in the original channel order, pruned entries 0.
+ *   keep_dev   : device uint8 n x k (original order), 1 = kept; may be NULL.
+ * Errors: DUO_EINVAL (NULL, sizes, pw_pct, block, dead context), DUO_ENOMEM,
+ * DUO_ECUDA.
+ */
+int duo_calib_prune(duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw, int pw_pct,
+                    int block, float* Wout_dev, uint8_t* keep_dev, void* stream);
+
 /* Frees a context (NULL is a no-op; an unknown or freed handle: DUO_EINVAL). */
 int duo_calib_free(duo_calib* h);
 

@@ -302,6 +302,292 @@ __global__ void score_kernel(const uint16_t* __restrict__ W, int64_t ldw, int k,
   S[r * k + p] = w * w * col[p];
 }
 
+// ---- Algorithm 1's column sweep ----
+
+constexpr int SWEEP_ROWS = 32;     // rows (one warp each) per CTA of the in-block sweep
+
+// W32[r][p] = W[r][perm[p]] (fp16 -> fp32, processing order).
+__global__ void load_permuted_kernel(const uint16_t* __restrict__ W, int64_t ldw, int k,
+                                     const int* __restrict__ perm, float* __restrict__ W32) {
+  const int p = blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t r = blockIdx.y;
+  if (p >= k) return;
+  W32[r * k + p] = __half2float(__ushort_as_half(W[r * ldw + perm[p]]));
+}
+
+// Monotone uint32 key of a float score (+0 and -0 map to the same key).
+__device__ __forceinline__ uint32_t score_key(float s) {
+  const uint32_t b = __float_as_uint(s + 0.f);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// Mask of one block (columns i .. i+bj-1, n rows): prune the `cnt` weights
+// with the lowest S = W^2 col (equal scores: lower flat index f = r*bj + c
+// first).  Multi-CTA radix select on the monotone keys: two 16-bit passes
+// with global histograms, each followed by a one-CTA pick of the digit, give
+// the cnt-th smallest key T and `want`, the number of elements equal to T to
+// prune; per-CTA tie counts and their scan then give every tie its rank in
+// flat order.  Elements are split into contiguous flat ranges of
+// SELM_PER_CTA, SELM_PER_THREAD consecutive ones per thread.
+constexpr int SELM_THREADS = 256;
+constexpr int SELM_PER_THREAD = 8;
+constexpr int SELM_PER_CTA = SELM_THREADS * SELM_PER_THREAD;
+constexpr int SEL_BINS16 = 1 << 16;
+
+struct SelState {
+  uint32_t prefix;   // T once both passes have run
+  uint32_t want;     // rank of T among the keys matching the prefix (1-based)
+};
+
+// Keys of the block in flat order, and the histogram of their high 16 bits.
+__global__ void __launch_bounds__(SELM_THREADS) sel_keys_kernel(const float* __restrict__ W32, int k, int i,
+                                                                int bj, int64_t N,
+                                                                const float* __restrict__ col,
+                                                                uint32_t* __restrict__ keys,
+                                                                uint32_t* __restrict__ hist) {
+  const int64_t f0 = (int64_t)blockIdx.x * SELM_PER_CTA + (int64_t)threadIdx.x * SELM_PER_THREAD;
+#pragma unroll
+  for (int e = 0; e < SELM_PER_THREAD; ++e) {
+    const int64_t f = f0 + e;
+    if (f < N) {
+      const int64_t r = f / bj;
+      const int c = (int)(f - r * bj);
+      const float w = W32[r * k + i + c];
+      const uint32_t key = score_key(w * w * col[i + c]);
+      keys[f] = key;
+      atomicAdd(&hist[key >> 16], 1u);
+    }
+  }
+}
+
+// Low 16 bits among the keys whose high bits equal the picked digit.
+__global__ void __launch_bounds__(SELM_THREADS) sel_low_hist_kernel(const uint32_t* __restrict__ keys, int64_t N,
+                                                                    const SelState* __restrict__ st,
+                                                                    uint32_t* __restrict__ hist) {
+  const uint32_t hi = st->prefix >> 16;
+  const int64_t f0 = (int64_t)blockIdx.x * SELM_PER_CTA + (int64_t)threadIdx.x * SELM_PER_THREAD;
+#pragma unroll
+  for (int e = 0; e < SELM_PER_THREAD; ++e) {
+    const int64_t f = f0 + e;
+    if (f < N && (keys[f] >> 16) == hi) atomicAdd(&hist[keys[f] & 0xFFFFu], 1u);
+  }
+}
+
+// One CTA: the digit where the cumulative count reaches `want`; clears the
+// histogram for the next pass.  pass 0 sets the high half of the prefix
+// (want = cnt on entry), pass 1 the low half.
+__global__ void __launch_bounds__(1024) sel_pick_kernel(uint32_t* __restrict__ hist, SelState* __restrict__ st,
+                                                        int pass, uint32_t cnt) {
+  __shared__ uint32_t part[1024];
+  __shared__ uint32_t s_digit, s_before;
+  const int t = threadIdx.x;
+  const uint32_t want = pass == 0 ? cnt : st->want;
+  if (t == 0) {   // stays so only when want == 0 (nothing to prune)
+    s_digit = 0;
+    s_before = 0;
+  }
+  uint32_t sum = 0;
+  for (int b = 0; b < 64; ++b) sum += hist[t * 64 + b];
+  part[t] = sum;
+  __syncthreads();
+  for (int o = 1; o < 1024; o <<= 1) {   // inclusive scan
+    const uint32_t v = t >= o ? part[t - o] : 0u;
+    __syncthreads();
+    part[t] += v;
+    __syncthreads();
+  }
+  const uint32_t incl = part[t], excl = incl - sum;
+  if (excl < want && want <= incl) {   // this thread's 64 bins hold the rank
+    uint32_t cum = excl;
+    int b = 0;
+    for (; b < 63; ++b) {
+      if (cum + hist[t * 64 + b] >= want) break;
+      cum += hist[t * 64 + b];
+    }
+    s_digit = (uint32_t)(t * 64 + b);
+    s_before = cum;
+  }
+  __syncthreads();
+  for (int b = 0; b < 64; ++b) hist[t * 64 + b] = 0u;
+  if (t == 0) {
+    if (pass == 0) {
+      st->prefix = s_digit << 16;
+    } else {
+      st->prefix |= s_digit;
+    }
+    st->want = want - s_before;
+  }
+}
+
+// Per CTA: how many keys equal T.
+__global__ void __launch_bounds__(SELM_THREADS) sel_tie_count_kernel(const uint32_t* __restrict__ keys, int64_t N,
+                                                                     const SelState* __restrict__ st,
+                                                                     uint32_t* __restrict__ ctacnt) {
+  __shared__ uint32_t part[SELM_THREADS / 32];
+  const uint32_t T = st->prefix;
+  const int64_t f0 = (int64_t)blockIdx.x * SELM_PER_CTA + (int64_t)threadIdx.x * SELM_PER_THREAD;
+  uint32_t c = 0;
+#pragma unroll
+  for (int e = 0; e < SELM_PER_THREAD; ++e) c += (f0 + e < N && keys[f0 + e] == T) ? 1u : 0u;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(FULL_MASK, c, o);
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t s2 = 0;
+    for (int w = 0; w < SELM_THREADS / 32; ++w) s2 += part[w];
+    ctacnt[blockIdx.x] = s2;
+  }
+}
+
+// One CTA: exclusive scan of the per-CTA tie counts (nb <= 65536).
+__global__ void __launch_bounds__(1024) sel_tie_scan_kernel(uint32_t* __restrict__ ctacnt, int nb) {
+  __shared__ uint32_t part[1024];
+  const int t = threadIdx.x;
+  const int per = (nb + 1023) / 1024;
+  uint32_t sum = 0;
+  for (int b = t * per; b < min(nb, t * per + per); ++b) sum += ctacnt[b];
+  part[t] = sum;
+  __syncthreads();
+  for (int o = 1; o < 1024; o <<= 1) {
+    const uint32_t v = t >= o ? part[t - o] : 0u;
+    __syncthreads();
+    part[t] += v;
+    __syncthreads();
+  }
+  uint32_t run = part[t] - sum;
+  for (int b = t * per; b < min(nb, t * per + per); ++b) {
+    const uint32_t c = ctacnt[b];
+    ctacnt[b] = run;
+    run += c;
+  }
+}
+
+// Keep flags: pruned iff key < T, or key == T with flat tie rank < want.
+__global__ void __launch_bounds__(SELM_THREADS) sel_mask_kernel(const uint32_t* __restrict__ keys, int64_t N,
+                                                                int k, int i, int bj,
+                                                                const SelState* __restrict__ st,
+                                                                const uint32_t* __restrict__ ctaoff,
+                                                                int none, uint8_t* __restrict__ keep) {
+  __shared__ uint32_t part[SELM_THREADS / 32];
+  const uint32_t T = st->prefix, want = st->want;
+  const int64_t f0 = (int64_t)blockIdx.x * SELM_PER_CTA + (int64_t)threadIdx.x * SELM_PER_THREAD;
+  uint32_t kv[SELM_PER_THREAD];
+  uint32_t c = 0;
+#pragma unroll
+  for (int e = 0; e < SELM_PER_THREAD; ++e) {
+    kv[e] = f0 + e < N ? keys[f0 + e] : 0xFFFFFFFFu;
+    c += (f0 + e < N && kv[e] == T) ? 1u : 0u;
+  }
+  // rank of this thread's first tie within the CTA
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  uint32_t inc = c;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t v = __shfl_up_sync(FULL_MASK, inc, o);
+    if (lane >= o) inc += v;
+  }
+  if (lane == 31) part[wid] = inc;
+  __syncthreads();
+  uint32_t wbefore = 0;
+  for (int w = 0; w < wid; ++w) wbefore += part[w];
+  uint32_t rank = ctaoff[blockIdx.x] + wbefore + inc - c;
+#pragma unroll
+  for (int e = 0; e < SELM_PER_THREAD; ++e) {
+    const int64_t f = f0 + e;
+    if (f < N) {
+      bool pruned = false;
+      if (!none) {
+        if (kv[e] < T) {
+          pruned = true;
+        } else if (kv[e] == T) {
+          pruned = rank < want;
+          ++rank;
+        }
+      }
+      const int64_t r = f / bj;
+      const int cc = (int)(f - r * bj);
+      keep[r * k + i + cc] = pruned ? 0 : 1;
+    }
+  }
+}
+
+// The block's sequential steps, one warp per row (lane l holds block
+// columns l, l+32, l+64, l+96): for column j, the owner lane broadcasts W_j
+// and its keep bit; P = W_j M_j, E_j = (W_j - P) / L_jj; later block
+// columns q get W_q -= E_j L_qj - W_j D_jq; W_j = P.  E and W_pre (each
+// column as it was at its step) are kept for the lazy update of the
+// trailing columns.  The block's L^T and D are staged in shared memory as
+// pairs {L_qj, D_jq} at [j][q], so a step's reads are consecutive per lane.
+__global__ void __launch_bounds__(SWEEP_ROWS * 32) block_sweep_kernel(float* __restrict__ W32, int n, int k,
+                                                                      int i, int bj,
+                                                                      const float* __restrict__ L,
+                                                                      const float* __restrict__ D,
+                                                                      const uint8_t* __restrict__ keep,
+                                                                      float* __restrict__ E,
+                                                                      float* __restrict__ Wpre) {
+  extern __shared__ __align__(128) uint8_t sm[];
+  float2* PD = reinterpret_cast<float2*>(sm);   // PD[j * bj + q] = {L[i+q][i+j], D[i+j][i+q]}
+  for (int e = threadIdx.x; e < bj * bj; e += blockDim.x) {
+    const int j = e / bj, q = e - j * bj;
+    PD[e] = make_float2(L[(size_t)(i + q) * k + (i + j)], D[(size_t)(i + j) * k + (i + q)]);
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * SWEEP_ROWS + warp;
+  if (r >= n) return;
+  float w[4];
+  uint32_t kb = 0;
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const int q = lane + 32 * u;
+    w[u] = q < bj ? W32[(size_t)r * k + i + q] : 0.f;
+    kb |= (q < bj && keep[(size_t)r * k + i + q]) ? (1u << u) : 0u;
+  }
+  for (int j = 0; j < bj; ++j) {
+    const int owner = j & 31, uj = j >> 5;
+    const float mine = uj == 0 ? w[0] : (uj == 1 ? w[1] : (uj == 2 ? w[2] : w[3]));
+    const float wj = __shfl_sync(FULL_MASK, mine, owner);
+    const uint32_t kj = __shfl_sync(FULL_MASK, (kb >> uj) & 1u, owner);
+    const float pj = kj ? wj : 0.f;
+    const float ej = (wj - pj) / PD[j * bj + j].x;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int q = lane + 32 * u;
+      if (q > j && q < bj) {
+        const float2 ld = PD[j * bj + q];
+        w[u] -= fmaf(ej, ld.x, -wj * ld.y);
+      }
+    }
+    if (lane == owner) {
+      if (uj == 0) w[0] = pj;
+      else if (uj == 1) w[1] = pj;
+      else if (uj == 2) w[2] = pj;
+      else w[3] = pj;
+      E[(size_t)r * bj + j] = ej;
+      Wpre[(size_t)r * bj + j] = wj;
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const int q = lane + 32 * u;
+    if (q < bj) W32[(size_t)r * k + i + q] = w[u];
+  }
+}
+
+// Back to the original channel order: Wout[r][perm[p]] = W32[r][p] and the
+// keep mask likewise.
+__global__ void store_unpermuted_kernel(const float* __restrict__ W32, const uint8_t* __restrict__ keepP,
+                                        int k, const int* __restrict__ perm, float* __restrict__ Wout,
+                                        uint8_t* __restrict__ keep_out) {
+  const int p = blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t r = blockIdx.y;
+  if (p >= k) return;
+  const int o = perm[p];
+  Wout[r * k + o] = W32[r * k + p];
+  if (keep_out != nullptr) keep_out[r * k + o] = keepP[r * k + p];
+}
+
 }  // namespace calib
 }  // namespace duo
 
@@ -333,6 +619,14 @@ struct duo_calib {
   size_t hwork_bytes;
   void* allocs[32];
   int nalloc;
+  // column sweep scratch, grown on demand: W32 (n x k fp32), keep (n x k),
+  // E and W_pre (n x 128 fp32 each)
+  float *sw_W32, *sw_E, *sw_Wpre;
+  uint8_t* sw_keep;
+  uint32_t *sw_keys, *sw_ctacnt;
+  int64_t sw_rows;
+  uint32_t* sel_hist;             // 65536 bins, zero between passes
+  duo::calib::SelState* sel_state;
 };
 
 namespace {
@@ -362,6 +656,12 @@ void release(duo_calib* h) {
   if (h->params) cusolverDnDestroyParams(h->params);
   if (h->solver) cusolverDnDestroy(h->solver);
   for (int i = 0; i < h->nalloc; ++i) cudaFree(h->allocs[i]);
+  cudaFree(h->sw_W32);
+  cudaFree(h->sw_E);
+  cudaFree(h->sw_Wpre);
+  cudaFree(h->sw_keep);
+  cudaFree(h->sw_keys);
+  cudaFree(h->sw_ctacnt);
   if (h->hwork) std::free(h->hwork);
   delete h;
 }
@@ -419,6 +719,9 @@ int duo_calib_create(int64_t k, int64_t m, void* stream, duo_calib** out) {
   if (e == cudaSuccess) e = alloc(h, &h->key_lo, (size_t)k);
   if (e == cudaSuccess) e = alloc(h, &h->perm, (size_t)k);
   if (e == cudaSuccess) e = alloc(h, &h->info, 2);
+  if (e == cudaSuccess) e = alloc(h, &h->sel_hist, (size_t)duo::calib::SEL_BINS16);
+  if (e == cudaSuccess) e = alloc(h, &h->sel_state, 1);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->sel_hist, 0, sizeof(uint32_t) * duo::calib::SEL_BINS16, st);
   if (e != cudaSuccess) return fail(map_cuda(e));
   // cuSOLVER workspace of the factorisation.
   size_t d1 = 0, h1 = 0;
@@ -608,6 +911,87 @@ int duo_calib_score(const duo_calib* h, const void* W_fp16_dev, int64_t n, int64
   const dim3 grid((k + 255) / 256, (unsigned)n);
   duo::calib::score_kernel<<<grid, 256, 0, static_cast<cudaStream_t>(stream)>>>(
       static_cast<const uint16_t*>(W_fp16_dev), ldw, k, h->perm, h->col, S_dev);
+  return map_cuda(cudaGetLastError());
+}
+
+int duo_calib_prune(duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw, int pw_pct, int block,
+                    float* Wout_dev, uint8_t* keep_dev, void* stream) {
+  if (h == nullptr || W_fp16_dev == nullptr || Wout_dev == nullptr || !calib_live(h)) return DUO_EINVAL;
+  if (n < 1 || n > 65535 || ldw < h->k || pw_pct < 0 || pw_pct > 100 || block < 1 || block > 128 ||
+      !aligned2(W_fp16_dev) || (reinterpret_cast<uintptr_t>(Wout_dev) & 3u) != 0)
+    return DUO_EINVAL;
+  using namespace duo::calib;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int k = (int)h->k;
+  cudaError_t e = cudaSuccess;
+  if (h->sw_rows < n) {   // grow the scratch (the stream's earlier work may still use it)
+    e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return map_cuda(e);
+    cudaFree(h->sw_W32);
+    cudaFree(h->sw_E);
+    cudaFree(h->sw_Wpre);
+    cudaFree(h->sw_keep);
+    cudaFree(h->sw_keys);
+    cudaFree(h->sw_ctacnt);
+    h->sw_W32 = h->sw_E = h->sw_Wpre = nullptr;
+    h->sw_keep = nullptr;
+    h->sw_keys = h->sw_ctacnt = nullptr;
+    h->sw_rows = 0;
+    const size_t nk = (size_t)n * k;
+    e = cudaMalloc(&h->sw_W32, nk * sizeof(float));
+    if (e == cudaSuccess) e = cudaMalloc(&h->sw_E, (size_t)n * 128 * sizeof(float));
+    if (e == cudaSuccess) e = cudaMalloc(&h->sw_Wpre, (size_t)n * 128 * sizeof(float));
+    if (e == cudaSuccess) e = cudaMalloc(&h->sw_keep, nk);
+    if (e == cudaSuccess) e = cudaMalloc(&h->sw_keys, (size_t)n * 128 * sizeof(uint32_t));
+    if (e == cudaSuccess)
+      e = cudaMalloc(&h->sw_ctacnt, ((size_t)n * 128 / SELM_PER_CTA + 1) * sizeof(uint32_t));
+    if (e != cudaSuccess) return map_cuda(e);
+    h->sw_rows = n;
+  }
+  float* W32 = h->sw_W32;
+  float* E = h->sw_E;
+  float* Wpre = h->sw_Wpre;
+  uint8_t* keepP = h->sw_keep;
+  const dim3 gk((k + 255) / 256, (unsigned)n);
+  load_permuted_kernel<<<gk, 256, 0, st>>>(static_cast<const uint16_t*>(W_fp16_dev), ldw, k, h->perm, W32);
+  const size_t ssm = (size_t)block * block * sizeof(float2);
+  e = cudaFuncSetAttribute(block_sweep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssm);
+  if (e != cudaSuccess) return map_cuda(e);
+  if (cublasSetStream(h->blas, st) != CUBLAS_STATUS_SUCCESS) return DUO_ECUDA;
+  const float one = 1.f, minus_one = -1.f;
+  for (int i = 0; i < k; i += block) {
+    const int bj = k - i < block ? k - i : block;
+    const int64_t cnt = (int64_t)n * bj * pw_pct / 100;
+    const int64_t N = (int64_t)n * bj;
+    const unsigned nb = (unsigned)((N + SELM_PER_CTA - 1) / SELM_PER_CTA);
+    sel_keys_kernel<<<nb, SELM_THREADS, 0, st>>>(W32, k, i, bj, N, h->col, h->sw_keys, h->sel_hist);
+    sel_pick_kernel<<<1, 1024, 0, st>>>(h->sel_hist, h->sel_state, 0, (uint32_t)cnt);
+    sel_low_hist_kernel<<<nb, SELM_THREADS, 0, st>>>(h->sw_keys, N, h->sel_state, h->sel_hist);
+    sel_pick_kernel<<<1, 1024, 0, st>>>(h->sel_hist, h->sel_state, 1, (uint32_t)cnt);
+    sel_tie_count_kernel<<<nb, SELM_THREADS, 0, st>>>(h->sw_keys, N, h->sel_state, h->sw_ctacnt);
+    sel_tie_scan_kernel<<<1, 1024, 0, st>>>(h->sw_ctacnt, (int)nb);
+    sel_mask_kernel<<<nb, SELM_THREADS, 0, st>>>(h->sw_keys, N, k, i, bj, h->sel_state, h->sw_ctacnt,
+                                                 cnt == 0 ? 1 : 0, keepP);
+    block_sweep_kernel<<<(unsigned)((n + SWEEP_ROWS - 1) / SWEEP_ROWS), SWEEP_ROWS * 32, ssm, st>>>(
+        W32, (int)n, k, i, bj, h->L, h->D, keepP, E, Wpre);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return map_cuda(e);
+    const int nt = k - i - bj;   // trailing columns
+    if (nt > 0) {
+      // Lazy batch: W_T -= E L_T,blk^T - W_pre D_blk,T.  Row-major buffers are
+      // column-major transposes: W_T^T (nt x n, ld k) += -(L^T)[blk, T]^T E^T
+      // + (D^T)[T, blk] W_pre^T.
+      int rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_T, CUBLAS_OP_N, nt, (int)n, bj, &minus_one,
+                                     h->L + i + (size_t)(i + bj) * k, CUDA_R_32F, k, E, CUDA_R_32F, bj, &one,
+                                     W32 + i + bj, CUDA_R_32F, k, kL_COMPUTE, CUBLAS_GEMM_DEFAULT));
+      if (rc != DUO_OK) return rc;
+      rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_N, CUBLAS_OP_N, nt, (int)n, bj, &one,
+                                 h->D + (i + bj) + (size_t)i * k, CUDA_R_32F, k, Wpre, CUDA_R_32F, bj, &one,
+                                 W32 + i + bj, CUDA_R_32F, k, kL_COMPUTE, CUBLAS_GEMM_DEFAULT));
+      if (rc != DUO_OK) return rc;
+    }
+  }
+  store_unpermuted_kernel<<<gk, 256, 0, st>>>(W32, keepP, k, h->perm, Wout_dev, keep_dev);
   return map_cuda(cudaGetLastError());
 }
 

@@ -65,6 +65,7 @@ def load_library(path: str | None = None):
     lib.duo_calib_status.argtypes = [vp, vp]
     lib.duo_calib_export.argtypes = [vp, i32, vp, i64, vp]
     lib.duo_calib_score.argtypes = [vp, vp, i64, i64, vp, vp]
+    lib.duo_calib_prune.argtypes = [vp, vp, i64, i64, i32, i32, vp, vp, vp]
     lib.duo_calib_free.argtypes = [vp]
     lib.duo_strerror.argtypes = [i32]
     lib.duo_strerror.restype = ctypes.c_char_p
@@ -72,7 +73,7 @@ def load_library(path: str | None = None):
                  "duo_packed_query", "duo_packed_export", "duo_device_status", "duo_abi_version",
                  "duo_pack_cmb_noalloc", "duo_sparsify_threshold", "duo_spmspv_threshold",
                  "duo_calib_create", "duo_calib_precompute", "duo_calib_status", "duo_calib_export",
-                 "duo_calib_score", "duo_calib_free"):
+                 "duo_calib_score", "duo_calib_free", "duo_calib_prune"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -327,6 +328,18 @@ class Calib:
         _check(load_library().duo_calib_score(self._h, W.data_ptr(), W.shape[0], W.stride(0),
                                               S.data_ptr(), _stream_ptr(stream)), "duo_calib_score")
         return S
+
+    def prune(self, W: torch.Tensor, pw_pct: int, block: int = 128, stream=None):
+        """Algorithm 1's column sweep: returns (pruned fp32 n x k, keep uint8
+        n x k), both in the original channel order."""
+        if W.dtype != torch.float16 or W.dim() != 2 or W.shape[1] != self.k or W.stride(1) != 1:
+            raise DuoError(DUO_EINVAL, "prune needs an n x k fp16 tensor with unit column stride")
+        out = torch.empty(W.shape[0], self.k, dtype=torch.float32, device=W.device)
+        keep = torch.empty(W.shape[0], self.k, dtype=torch.uint8, device=W.device)
+        _check(load_library().duo_calib_prune(self._h, W.data_ptr(), W.shape[0], W.stride(0), int(pw_pct),
+                                              int(block), out.data_ptr(), keep.data_ptr(),
+                                              _stream_ptr(stream)), "duo_calib_prune")
+        return out, keep
 
     def free(self):
         if self._h:

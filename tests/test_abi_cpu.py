@@ -32,7 +32,7 @@ def test_header_declares_the_boundary():
               "duo_strerror", "duo_packed_query", "duo_packed_export", "duo_device_status",
               "duo_abi_version", "duo_sparsify_threshold", "duo_spmspv_threshold",
               "duo_calib_create", "duo_calib_precompute", "duo_calib_status", "duo_calib_query",
-              "duo_calib_export", "duo_calib_score", "duo_calib_free"):
+              "duo_calib_export", "duo_calib_score", "duo_calib_free", "duo_calib_prune"):
         assert n in names
 
 
@@ -147,5 +147,8 @@ def test_calib_argument_validation(lib):
     assert lib.duo_calib_score(FAKE, FAKE, 4, 8, FAKE, None) == EINVAL
     assert lib.duo_calib_status(FAKE, None) == EINVAL
     assert lib.duo_calib_export(FAKE, 0, FAKE, 32, None) == EINVAL
+    lib.duo_calib_prune.argtypes = [vp, vp, i64, i64, ctypes.c_int, ctypes.c_int, vp, vp, vp]
+    assert lib.duo_calib_prune(FAKE, FAKE, 4, 8, 50, 128, FAKE, None, None) == EINVAL
+    assert lib.duo_calib_prune(None, FAKE, 4, 8, 50, 128, FAKE, None, None) == EINVAL
     assert lib.duo_calib_free(FAKE) == EINVAL
     assert lib.duo_calib_free(None) == 0
