@@ -149,3 +149,35 @@ def test_sweep_full_size_layer(duo):
     assert (kmask != mref).sum() <= 2e-3 * n * k
     same = (kmask == mref).all(axis=1)
     _close("W (rows with identical masks)", out[same], Wref[same], TOL_FACTOR)
+
+
+def test_prune_then_pack_then_decode(duo):
+    """The two halves together: calibrate and prune a layer on the GPU
+    (Algorithm 1), pack the pruned weight, and run the fused dual-sparse
+    product on a new input: y matches the oracle's product with the same
+    pruned weight within the decode tolerance."""
+    n, k, m = 1536, 512, 700
+    X = _inputs(k, m, 41)
+    rng = np.random.default_rng(42)
+    W = (rng.standard_normal((n, k)) * 0.02).astype(np.float16)
+    c = duo.Calib(k, m)
+    c.precompute(torch.from_numpy(np.ascontiguousarray(X.T)).cuda(), k // 2)
+    out, keep = c.prune(torch.from_numpy(W).cuda(), 50, 128)
+    assert c.status() == 0
+    c.free()
+    Wp = out.to(torch.float16)
+    # a kept weight that rounds to zero in fp16 would read as pruned: keep it
+    # at the smallest fp16 magnitude instead
+    tiny = (Wp == 0) & (keep == 1)
+    Wp[tiny] = torch.where(out[tiny] >= 0, 2.0 ** -24, -(2.0 ** -24)).to(torch.float16)
+    assert int((Wp != 0).sum()) == int(keep.sum()) == n * k // 2
+    h = duo.duo_pack(Wp, "bitmask")
+    x = torch.from_numpy(rng.laplace(0, 1, size=k).astype(np.float16))
+    kk = k // 2
+    y = duo.duo_spmspv(h, x.cuda(), kk).cpu().numpy().astype(np.float64)
+    Wn = Wp.cpu().numpy()
+    y_ref = orc.oracle_spmspv(Wn, x.numpy(), kk)
+    K, _ = orc.oracle_sparsify(x.numpy(), kk)
+    assert np.all(np.abs(y - y_ref) <= orc.tolerance_rows(Wn, x.numpy(), K))
+    h.free()
+    assert duo.duo_device_status() == 0
