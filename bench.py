@@ -612,16 +612,42 @@ def run_calib(duo, reps):
 
 
 def run_e2e(duo, shape, layers, args, breq_mean):
-    """Public-API calls with host (pinned) inputs copied in and outputs read
-    back every step; no graph (this is the call a user makes)."""
+    """End to end through the public API: every step copies that layer's
+    inputs from pinned host memory to the device, runs the four stage calls
+    and copies every output back.  Measured two ways: with duo.StepGraph
+    (the step captured once, one replay call per step, one copy each way:
+    the serving call) as the reported value, and with the individual calls
+    and per-tensor copies issued eagerly from Python each step."""
     L = len(layers)
     hx = [{s: layers[l]["x"][s].cpu().pin_memory() for s in STAGE_SRC} for l in range(L)]
     hy = [{p: torch.empty(shape.O(p), dtype=torch.float32).pin_memory() for p in layers[l]["y"]}
           for l in range(L)]
     h2d = sum(t.numel() * 2 for t in hx[0].values())
     d2h = sum(t.numel() * 4 for t in hy[0].values())
+    n = min(args.steps, 2000)
 
-    def step(i):
+    def timed(step):
+        for i in range(min(args.warmup, 50)):
+            step(i)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for i in range(n):
+            step(i)
+        torch.cuda.synchronize()
+        return time.perf_counter() - t0
+
+    plans = []
+    for l in range(L):
+        plan = duo.StepGraph([{"h": [layers[l]["h"][p] for p in st], "k": k_of(shape.I(st[0]), args.px)}
+                              for st in STAGES])
+        for si, src in enumerate(STAGE_SRC):
+            plan.x_host(si).copy_(hx[l][src])   # the layer's inputs, written once on the host
+        plans.append(plan)
+    h2d_graph = sum(p._xh.numel() * 2 for p in plans[:1])
+    d2h_graph = sum(p._yh.numel() * 4 for p in plans[:1])
+    t_graph = timed(lambda i: plans[i % L].run())
+
+    def eager(i):
         l = i % L
         lay = layers[l]
         for s in STAGE_SRC:
@@ -629,18 +655,14 @@ def run_e2e(duo, shape, layers, args, breq_mean):
         stage_calls(duo, shape, lay, args.px)()
         for p in lay["y"]:
             hy[l][p].copy_(lay["y"][p], non_blocking=True)
-
-    n = min(args.steps, 2000)
-    for i in range(min(args.warmup, 50)):
-        step(i)
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    for i in range(n):
-        step(i)
-    torch.cuda.synchronize()
-    t = time.perf_counter() - t0
-    return {"value": breq_mean * n / t / 1e9, "unit": "GB/s", "us_per_layer": t / n * 1e6,
-            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n}
+    t_eager = timed(eager)
+    del plans
+    return {"value": breq_mean * n / t_graph / 1e9, "unit": "GB/s", "us_per_layer": t_graph / n * 1e6,
+            "h2d_bytes_per_step": h2d_graph, "d2h_bytes_per_step": d2h_graph, "steps": n,
+            "api": "duo.StepGraph: one H2D copy of the step's inputs, the 4 stage calls, one D2H copy "
+                   "of all outputs, replayed as one graph per step",
+            "eager_calls": {"value": breq_mean * n / t_eager / 1e9, "us_per_layer": t_eager / n * 1e6,
+                            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}}
 
 
 def run_dense(shape, layers, reps):

@@ -351,3 +351,66 @@ class Calib:
             self.free()
         except Exception:
             pass
+
+
+class StepGraph:
+    """A decode step of several dual-sparse products, captured once as a
+    CUDA graph and replayed with one call: one host -> device copy of all the
+    step's inputs, the products back to back, one device -> host copy of all
+    outputs.
+
+    ``stages`` is a list of dicts: ``h`` (a Packed, or a list of up to 4
+    sharing one input) and ``k`` (kept channels).  The object owns one pinned
+    host buffer for the inputs and one for the outputs; ``x_host(i)`` and
+    ``y_host(i, j)`` are views of them (fp16 input of stage i, fp32 output of
+    its j-th product).  Write the next inputs into the x_host views before
+    :meth:`run`; the outputs are in the y_host views once the stream has
+    finished."""
+
+    def __init__(self, stages, stream=None):
+        self._stages = []
+        xoff = yoff = 0
+        for st in stages:
+            hs = list(st["h"]) if isinstance(st["h"], (list, tuple)) else [st["h"]]
+            I = hs[0].inp
+            yo = []
+            for h in hs:
+                yo.append((yoff, h.out))
+                yoff += (h.out + 3) // 4 * 4            # 16-byte aligned outputs
+            self._stages.append((hs, int(st["k"]), xoff, I, yo))
+            xoff += (I + 7) // 8 * 8                     # 16-byte aligned inputs
+        self._xh = torch.zeros(max(xoff, 8), dtype=torch.float16).pin_memory()
+        self._yh = torch.zeros(max(yoff, 4), dtype=torch.float32).pin_memory()
+        self._xd = torch.zeros_like(self._xh, device="cuda")
+        self._yd = torch.zeros_like(self._yh, device="cuda")
+        s = torch.cuda.Stream() if stream is None else stream
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):   # one eager pass (library state, launch attributes)
+            self._enqueue()
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            self._enqueue()
+
+    def x_host(self, i):
+        _, _, off, I, _ = self._stages[i]
+        return self._xh[off:off + I]
+
+    def y_host(self, i, j=0):
+        off, O = self._stages[i][4][j]
+        return self._yh[off:off + O]
+
+    def _enqueue(self):
+        self._xd.copy_(self._xh, non_blocking=True)
+        for hs, k, xo, I, yo in self._stages:
+            x = self._xd[xo:xo + I]
+            ys = [self._yd[o:o + O] for o, O in yo]
+            if len(hs) == 1:
+                duo_spmspv(hs[0], x, k, y=ys[0])
+            else:
+                duo_spmspv_multi(hs, x, k, ys=ys)
+        self._yh.copy_(self._yd, non_blocking=True)
+
+    def run(self):
+        self.graph.replay()

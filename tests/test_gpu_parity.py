@@ -386,3 +386,33 @@ except duo.DuoError as e:
         out = r.stdout.split()
         assert out[0] == "CODE" and int(out[1]) == -2, r.stdout
         assert int(out[3]) <= 2 * 1024 * 1024, f"leak after injected failure {n}: {out[3]} bytes"
+
+
+def test_step_graph_copies_and_products(duo):
+    """duo.StepGraph: a captured step (pinned-host inputs in, outputs out)
+    gives the oracle's y, for new inputs written before each run; two stages,
+    one of them a shared-input pair."""
+    d = duo
+    rng = np.random.default_rng(77)
+    I1, I2 = 1000, 333
+    Ws = [(rng.standard_normal((O, I1)) * 0.02).astype(np.float16) for O in (700, 1300)]
+    W2 = (rng.standard_normal((517, I2)) * 0.02).astype(np.float16)
+    for W in Ws + [W2]:
+        W[rng.random(W.shape) < 0.5] = 0
+    hs = [d.duo_pack(torch.from_numpy(W).cuda(), "bitmask") for W in Ws]
+    h2 = d.duo_pack(torch.from_numpy(W2).cuda(), "bitmask")
+    plan = d.StepGraph([{"h": hs, "k": 400}, {"h": h2, "k": 100}])
+    for trial in range(3):
+        x1 = rng.laplace(0, 1, size=I1).astype(np.float16)
+        x2 = rng.laplace(0, 1, size=I2).astype(np.float16)
+        plan.x_host(0).copy_(torch.from_numpy(x1))
+        plan.x_host(1).copy_(torch.from_numpy(x2))
+        plan.run()
+        torch.cuda.synchronize()
+        for (W, x, kk, y) in [(Ws[0], x1, 400, plan.y_host(0, 0)), (Ws[1], x1, 400, plan.y_host(0, 1)),
+                              (W2, x2, 100, plan.y_host(1))]:
+            K, _ = orc.oracle_sparsify(x, kk)
+            err = np.abs(y.numpy().astype(np.float64) - orc.oracle_spmspv(W, x, kk))
+            assert np.all(err <= orc.tolerance_rows(W, x, K)), trial
+    for h in hs + [h2]:
+        h.free()
