@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--profile", action="store_true",
                     help="small case for ncu: 2 layers, a few direct (ungraphed) layer steps")
+    ap.add_argument("--profile-coded", action="store_true",
+                    help="small case for ncu: one 7B layer's four stages once per format (fp16, 8-bit, 4-bit)")
     ap.add_argument("--profile-calib", action="store_true",
                     help="small case for ncu: `--steps` calibration precomputes of a 4096-channel layer")
     ap.add_argument("--stack", default=None,
@@ -707,6 +709,30 @@ def run_profile(args):
     print("profile workload done", flush=True)
 
 
+def run_profile_coded(args):
+    """One LLaMA-2-7B-shaped layer packed as fp16 records and as 8- and
+    4-bit RTN codes; the four stages once per format, in that order (12
+    fused launches), for profiler captures."""
+    torch.cuda.set_device(0)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2506_20194_gb300 import duo, synth
+    duo.load_library()
+    wl = synth.WORKLOADS[WORKLOAD]
+    shape = wl["shape"]
+    W = {p: synth.layer_weight(wl, p, layer=0, device="cuda") for p in synth.PROJS}
+    X = {s: synth.layer_input(wl, s, layer=0, device="cuda") for s in STAGE_SRC}
+    for fmt in ("bitmask", "bitmask_q8", "bitmask_q4"):
+        hs = {p: duo.duo_pack(W[p], fmt) for p in W}
+        for st, src in zip(STAGES, STAGE_SRC):
+            duo.duo_spmspv_multi([hs[p] for p in st], X[src], k_of(shape.I(st[0]), args.px))
+        torch.cuda.synchronize()
+        for h in hs.values():
+            h.free()
+    assert duo.duo_device_status() == duo.DUO_OK
+    print("profile workload done", flush=True)
+
+
 def run_profile_calib(args):
     """Calibration precompute for profiler captures: one 4096-channel layer
     from 2048 tokens, one warm-up and `--steps` precomputes, no graphs."""
@@ -796,6 +822,8 @@ def main():
         run_profile(args)
     elif args.profile_calib:
         run_profile_calib(args)
+    elif args.profile_coded:
+        run_profile_coded(args)
     elif args.stack is not None:
         run_stack(args)
     elif args.impl == "reference":

@@ -199,3 +199,22 @@ def test_spmspv_q_graph_replay(duo):
     _check_y(y.cpu().numpy(), Wd, x2.numpy(), K2, "graph replay new x")
     h.free()
     assert duo.duo_device_status() == 0
+
+
+def test_coded_launch_needs_a_run_per_sm(duo):
+    """More (product, segment) runs than SMs: the coded formats refuse the
+    launch on the host (DUO_ERANGE) instead of falling back."""
+    props = torch.cuda.get_device_properties(0)
+    O, I = (props.multi_processor_count + 1) * 1024, 64
+    W = torch.zeros(O, I, dtype=torch.float16)
+    W[::3, ::2] = 0.01
+    h = duo.duo_pack(W.cuda(), "bitmask_q8")
+    x = _laplace(I, 1).cuda()
+    with pytest.raises(duo.DuoError) as ei:
+        duo.duo_spmspv(h, x, I // 2)
+    assert ei.value.code == duo.DUO_ERANGE
+    with pytest.raises(duo.DuoError) as ei:
+        duo.duo_spmspv_threshold(h, x, 0.5)
+    assert ei.value.code == duo.DUO_ERANGE
+    h.free()
+    assert duo.duo_device_status() == 0
