@@ -218,3 +218,26 @@ def test_coded_launch_needs_a_run_per_sm(duo):
     assert ei.value.code == duo.DUO_ERANGE
     h.free()
     assert duo.duo_device_status() == 0
+
+
+def test_listed_out_of_group_order_is_rejected(duo):
+    """A coded launch streams grid tables in group order, so a kept list
+    whose ids decrease across 128-channel groups is rejected on the device
+    (duo_device_status: DUO_EFORMAT); the next call on the same handle
+    works."""
+    O, I = 2048, 1024
+    W = _weight(O, I, 0.5, 5, "gauss")
+    h = duo.duo_pack(W.cuda(), "bitmask_q8")
+    x = _laplace(I, 6)
+    k = 300
+    ids = np.arange(I - 1, I - 1 - k, -1).astype(np.uint16)          # descending
+    kidx = torch.from_numpy(ids.view(np.int16).copy()).cuda()
+    kval = x[torch.from_numpy(ids.astype(np.int64))].cuda()
+    duo.duo_spmspv(h, None, k, kept_idx=kidx, kept_val=kval)
+    assert duo.duo_device_status() == duo.DUO_EFORMAT
+    y = duo.duo_spmspv(h, x.cuda(), k)                                # fused: fine again
+    torch.cuda.synchronize()
+    K, _ = orc.oracle_sparsify(x.numpy(), k)
+    _check_y(y.cpu().numpy(), orc.oracle_dequantize(W.numpy(), 8), x.numpy(), K, "after rejection")
+    assert duo.duo_device_status() == 0
+    h.free()
