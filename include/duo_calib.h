@@ -121,8 +121,9 @@ int duo_calib_score(const duo_calib* h, const void* W_fp16_dev, int64_t n, int64
  * W_q -= E_j L_qj - W_j D_jq (within the block at once, for the columns
  * after the block in one lazy product that uses each W_j as it was at its
  * step); finally W_j = P_j.  Asynchronous; the context keeps scratch of
- * about n k (4 + 1) bytes, grown when a call needs more rows (growing waits
- * for the stream).
+ * about n k (4 + 1) + n 2 KiB bytes, grown when a call needs more rows
+ * (growing waits for the stream), and 8 k^2 bytes for the lazy products'
+ * operand (interleaved -L and D^T), rebuilt after each precompute.
  *   W_fp16_dev : device fp16, n x k row-major (leading dimension ldw), the
  *                dense weight in the ORIGINAL channel order.
  *   pw_pct     : weight sparsity in percent, 0..100.   block : 1..128 (the

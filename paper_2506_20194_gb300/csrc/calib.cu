@@ -323,98 +323,122 @@ __device__ __forceinline__ uint32_t score_key(float s) {
 
 // Mask of one block (columns i .. i+bj-1, n rows): prune the `cnt` weights
 // with the lowest S = W^2 col (equal scores: lower flat index f = r*bj + c
-// first).  Multi-CTA radix select on the monotone keys: two 16-bit passes
-// with global histograms, each followed by a one-CTA pick of the digit, give
-// the cnt-th smallest key T and `want`, the number of elements equal to T to
-// prune; per-CTA tie counts and their scan then give every tie its rank in
-// flat order.  Elements are split into contiguous flat ranges of
+// first).  Multi-CTA radix select on the monotone keys: three passes of 11,
+// 11 and 10 bits, each a histogram (per-CTA in shared memory, merged into a
+// global one over the non-empty bins) followed by a one-CTA pick of the
+// digit, give the cnt-th smallest key T and `want`, the number of elements
+// equal to T to prune; per-CTA tie counts and their scan then give every tie
+// its rank in flat order.  Elements are split into contiguous flat ranges of
 // SELM_PER_CTA, SELM_PER_THREAD consecutive ones per thread.
 constexpr int SELM_THREADS = 256;
 constexpr int SELM_PER_THREAD = 8;
 constexpr int SELM_PER_CTA = SELM_THREADS * SELM_PER_THREAD;
-constexpr int SEL_BINS16 = 1 << 16;
+constexpr int SEL_BINS16 = 2048;   // the largest digit (11 bits)
 
 struct SelState {
-  uint32_t prefix;   // T once both passes have run
+  uint32_t prefix;   // T once all passes have run
   uint32_t want;     // rank of T among the keys matching the prefix (1-based)
 };
 
-// Keys of the block in flat order, and the histogram of their high 16 bits.
-__global__ void __launch_bounds__(SELM_THREADS) sel_keys_kernel(const float* __restrict__ W32, int k, int i,
-                                                                int bj, int64_t N,
+__device__ __forceinline__ int sel_shift(int pass) { return pass == 0 ? 21 : (pass == 1 ? 10 : 0); }
+__device__ __forceinline__ uint32_t sel_bins(int pass) { return pass == 2 ? 1024u : 2048u; }
+
+// Keys of the block in flat order (f = r*bj + c), and the histogram of their
+// top 11 bits.  Grid-strided; (r, c) advance by the stride without a division.
+__global__ void __launch_bounds__(SELM_THREADS) sel_keys_kernel(const float* __restrict__ W32, int n, int k,
+                                                                int i, int bj,
                                                                 const float* __restrict__ col,
                                                                 uint32_t* __restrict__ keys,
                                                                 uint32_t* __restrict__ hist) {
-  const int64_t f0 = (int64_t)blockIdx.x * SELM_PER_CTA + (int64_t)threadIdx.x * SELM_PER_THREAD;
-#pragma unroll
-  for (int e = 0; e < SELM_PER_THREAD; ++e) {
-    const int64_t f = f0 + e;
-    if (f < N) {
-      const int64_t r = f / bj;
-      const int c = (int)(f - r * bj);
-      const float w = W32[r * k + i + c];
-      const uint32_t key = score_key(w * w * col[i + c]);
-      keys[f] = key;
-      atomicAdd(&hist[key >> 16], 1u);
+  __shared__ uint32_t h[SEL_BINS16];
+  for (int b = threadIdx.x; b < SEL_BINS16; b += SELM_THREADS) h[b] = 0u;
+  __syncthreads();
+  const int64_t N = (int64_t)n * bj;
+  const int stride = (int)gridDim.x * SELM_THREADS;
+  const int dr = stride / bj, dc = stride - dr * bj;
+  const int f0 = (int)blockIdx.x * SELM_THREADS + (int)threadIdx.x;
+  int64_t r = f0 / bj;
+  int c = f0 - (int)r * bj;
+  for (int64_t f = f0; f < N; f += stride) {
+    const float w = W32[r * k + i + c];
+    const uint32_t key = score_key(w * w * col[i + c]);
+    keys[f] = key;
+    atomicAdd(&h[key >> 21], 1u);
+    r += dr;
+    c += dc;
+    if (c >= bj) {
+      c -= bj;
+      ++r;
     }
   }
+  __syncthreads();
+  for (int b = threadIdx.x; b < SEL_BINS16; b += SELM_THREADS)
+    if (h[b]) atomicAdd(&hist[b], h[b]);
 }
 
-// Low 16 bits among the keys whose high bits equal the picked digit.
-__global__ void __launch_bounds__(SELM_THREADS) sel_low_hist_kernel(const uint32_t* __restrict__ keys, int64_t N,
-                                                                    const SelState* __restrict__ st,
-                                                                    uint32_t* __restrict__ hist) {
-  const uint32_t hi = st->prefix >> 16;
-  const int64_t f0 = (int64_t)blockIdx.x * SELM_PER_CTA + (int64_t)threadIdx.x * SELM_PER_THREAD;
-#pragma unroll
-  for (int e = 0; e < SELM_PER_THREAD; ++e) {
-    const int64_t f = f0 + e;
-    if (f < N && (keys[f] >> 16) == hi) atomicAdd(&hist[keys[f] & 0xFFFFu], 1u);
+// Histogram of pass 1 or 2's digit among the keys matching the prefix.
+__global__ void __launch_bounds__(SELM_THREADS) sel_hist_kernel(const uint32_t* __restrict__ keys, int64_t N,
+                                                                const SelState* __restrict__ st, int pass,
+                                                                uint32_t* __restrict__ hist) {
+  __shared__ uint32_t h[SEL_BINS16];
+  for (int b = threadIdx.x; b < SEL_BINS16; b += SELM_THREADS) h[b] = 0u;
+  __syncthreads();
+  const int sh = sel_shift(pass);
+  const uint32_t hi = st->prefix >> (sh + (pass == 1 ? 11 : 10));
+  const uint32_t dmask = sel_bins(pass) - 1u;
+  for (int64_t f = (int64_t)blockIdx.x * SELM_THREADS + threadIdx.x; f < N; f += (int64_t)gridDim.x * SELM_THREADS) {
+    const uint32_t key = keys[f];
+    if ((key >> (sh + (pass == 1 ? 11 : 10))) == hi) atomicAdd(&h[(key >> sh) & dmask], 1u);
   }
+  __syncthreads();
+  for (int b = threadIdx.x; b < SEL_BINS16; b += SELM_THREADS)
+    if (h[b]) atomicAdd(&hist[b], h[b]);
 }
 
-// One CTA: the digit where the cumulative count reaches `want`; clears the
-// histogram for the next pass.  pass 0 sets the high half of the prefix
-// (want = cnt on entry), pass 1 the low half.
+// One CTA: the digit where the cumulative count reaches `want` (pass 0:
+// want = cnt), the prefix extended by it; clears the histogram.
 __global__ void __launch_bounds__(1024) sel_pick_kernel(uint32_t* __restrict__ hist, SelState* __restrict__ st,
                                                         int pass, uint32_t cnt) {
-  __shared__ uint32_t part[1024];
+  __shared__ uint32_t wsum[32];
   __shared__ uint32_t s_digit, s_before;
-  const int t = threadIdx.x;
+  const int t = threadIdx.x, lane = t & 31, wid = t >> 5;
   const uint32_t want = pass == 0 ? cnt : st->want;
   if (t == 0) {   // stays so only when want == 0 (nothing to prune)
     s_digit = 0;
     s_before = 0;
   }
-  uint32_t sum = 0;
-  for (int b = 0; b < 64; ++b) sum += hist[t * 64 + b];
-  part[t] = sum;
-  __syncthreads();
-  for (int o = 1; o < 1024; o <<= 1) {   // inclusive scan
-    const uint32_t v = t >= o ? part[t - o] : 0u;
-    __syncthreads();
-    part[t] += v;
-    __syncthreads();
+  // thread t: bins 2t, 2t+1 (2048 bins; pass 2 uses the first 1024)
+  const uint2 hv = reinterpret_cast<const uint2*>(hist)[t];
+  const uint32_t sum = hv.x + hv.y;
+  uint32_t inc = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t v = __shfl_up_sync(FULL_MASK, inc, o);
+    if (lane >= o) inc += v;
   }
-  const uint32_t incl = part[t], excl = incl - sum;
-  if (excl < want && want <= incl) {   // this thread's 64 bins hold the rank
-    uint32_t cum = excl;
-    int b = 0;
-    for (; b < 63; ++b) {
-      if (cum + hist[t * 64 + b] >= want) break;
-      cum += hist[t * 64 + b];
+  if (lane == 31) wsum[wid] = inc;
+  __syncthreads();
+  if (wid == 0) {
+    uint32_t v = wsum[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t u = __shfl_up_sync(FULL_MASK, v, o);
+      if (lane >= o) v += u;
     }
-    s_digit = (uint32_t)(t * 64 + b);
-    s_before = cum;
+    wsum[lane] = v;
   }
   __syncthreads();
-  for (int b = 0; b < 64; ++b) hist[t * 64 + b] = 0u;
+  const uint32_t excl = (wid > 0 ? wsum[wid - 1] : 0u) + inc - sum;
+  if (excl < want && want <= excl + sum) {   // this thread's two bins hold the rank
+    const bool first = excl + hv.x >= want;
+    s_digit = 2u * (uint32_t)t + (first ? 0u : 1u);
+    s_before = first ? excl : excl + hv.x;
+  }
+  __syncthreads();
+  reinterpret_cast<uint2*>(hist)[t] = make_uint2(0u, 0u);
   if (t == 0) {
-    if (pass == 0) {
-      st->prefix = s_digit << 16;
-    } else {
-      st->prefix |= s_digit;
-    }
+    const uint32_t d = s_digit << sel_shift(pass);
+    st->prefix = pass == 0 ? d : (st->prefix | d);
     st->want = want - s_before;
   }
 }
@@ -513,65 +537,94 @@ __global__ void __launch_bounds__(SELM_THREADS) sel_mask_kernel(const uint32_t* 
 }
 
 // The block's sequential steps, one warp per row (lane l holds block
-// columns l, l+32, l+64, l+96): for column j, the owner lane broadcasts W_j
-// and its keep bit; P = W_j M_j, E_j = (W_j - P) / L_jj; later block
-// columns q get W_q -= E_j L_qj - W_j D_jq; W_j = P.  E and W_pre (each
-// column as it was at its step) are kept for the lazy update of the
-// trailing columns.  The block's L^T and D are staged in shared memory as
-// pairs {L_qj, D_jq} at [j][q], so a step's reads are consecutive per lane.
-__global__ void __launch_bounds__(SWEEP_ROWS * 32) block_sweep_kernel(float* __restrict__ W32, int n, int k,
-                                                                      int i, int bj,
-                                                                      const float* __restrict__ L,
-                                                                      const float* __restrict__ D,
-                                                                      const uint8_t* __restrict__ keep,
-                                                                      float* __restrict__ E,
-                                                                      float* __restrict__ Wpre) {
+// columns l, l+32, l+64, l+96): for column j, the owner lane broadcasts W_j;
+// P = W_j M_j, E_j = (W_j - P) / L_jj; later block columns q get
+// W_q -= E_j L_qj - W_j D_jq; W_j = P.  The pairs {E_j, W_j as it was at its
+// step} are kept for the lazy update of the trailing columns.  The block's
+// coefficients come from Z (Z[q][j] = {-L_qj, D_jq}) into shared memory as
+// T[j][q] (pitch SWEEP_TP), zero for q <= j, so that every lane applies
+// every step to its columns without a predicate; L_jj separately.  The keep
+// bits of a row are four warp-uniform ballots.  Rows per CTA: launch-time
+// (warps of the block), one CTA per SM.
+constexpr int SWEEP_TP = 129;   // float2 pitch of T's rows (q), padded against bank conflicts
+constexpr size_t SWEEP_SMEM = (size_t)128 * SWEEP_TP * sizeof(float2) + 128 * sizeof(float);
+
+__global__ void __launch_bounds__(1024, 1) block_sweep_kernel(float* __restrict__ W32, int n, int k, int i,
+                                                              int bj, const float2* __restrict__ Z,
+                                                              const float* __restrict__ L,
+                                                              const uint8_t* __restrict__ keep,
+                                                              float2* __restrict__ EW) {
   extern __shared__ __align__(128) uint8_t sm[];
-  float2* PD = reinterpret_cast<float2*>(sm);   // PD[j * bj + q] = {L[i+q][i+j], D[i+j][i+q]}
-  for (int e = threadIdx.x; e < bj * bj; e += blockDim.x) {
-    const int j = e / bj, q = e - j * bj;
-    PD[e] = make_float2(L[(size_t)(i + q) * k + (i + j)], D[(size_t)(i + j) * k + (i + q)]);
+  float2* T = reinterpret_cast<float2*>(sm);
+  float* Ld = reinterpret_cast<float*>(sm + (size_t)128 * SWEEP_TP * sizeof(float2));
+  for (int e = threadIdx.x; e < 128 * 128; e += blockDim.x) {   // j fastest: Z's rows are read in order
+    const int q = e >> 7, j = e & 127;
+    T[j * SWEEP_TP + q] = (q > j && q < bj) ? Z[(size_t)(i + q) * k + i + j] : make_float2(0.f, 0.f);
   }
+  for (int t = threadIdx.x; t < 128; t += blockDim.x) Ld[t] = t < bj ? L[(size_t)(i + t) * (k + 1)] : 1.f;
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int r = blockIdx.x * SWEEP_ROWS + warp;
+  const int r = blockIdx.x * (blockDim.x >> 5) + warp;
   if (r >= n) return;
   float w[4];
-  uint32_t kb = 0;
+  uint32_t km[4];
+  float2 ew[4];
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
     const int q = lane + 32 * u;
     w[u] = q < bj ? W32[(size_t)r * k + i + q] : 0.f;
-    kb |= (q < bj && keep[(size_t)r * k + i + q]) ? (1u << u) : 0u;
+    km[u] = __ballot_sync(FULL_MASK, q < bj && keep[(size_t)r * k + i + q] != 0);
+    ew[u] = make_float2(0.f, 0.f);
   }
-  for (int j = 0; j < bj; ++j) {
-    const int owner = j & 31, uj = j >> 5;
-    const float mine = uj == 0 ? w[0] : (uj == 1 ? w[1] : (uj == 2 ? w[2] : w[3]));
-    const float wj = __shfl_sync(FULL_MASK, mine, owner);
-    const uint32_t kj = __shfl_sync(FULL_MASK, (kb >> uj) & 1u, owner);
-    const float pj = kj ? wj : 0.f;
-    const float ej = (wj - pj) / PD[j * bj + j].x;
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int q = lane + 32 * u;
-      if (q > j && q < bj) {
-        const float2 ld = PD[j * bj + q];
-        w[u] -= fmaf(ej, ld.x, -wj * ld.y);
+  for (int uj = 0; uj < 4; ++uj) {
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+      const int j = uj * 32 + jj;
+      if (j < bj) {
+        const float wj = __shfl_sync(FULL_MASK, w[uj], jj);
+        const bool kj = ((km[uj] >> jj) & 1u) != 0u;
+        const float ej = kj ? 0.f : wj / Ld[j];
+        const float2* Tj = T + j * SWEEP_TP + lane;
+#pragma unroll
+        for (int u = uj; u < 4; ++u) {
+          const float2 z = Tj[32 * u];
+          w[u] = fmaf(ej, z.x, fmaf(wj, z.y, w[u]));
+        }
+        if (lane == jj) {
+          w[uj] = kj ? wj : 0.f;
+          ew[uj] = make_float2(ej, wj);
+        }
       }
-    }
-    if (lane == owner) {
-      if (uj == 0) w[0] = pj;
-      else if (uj == 1) w[1] = pj;
-      else if (uj == 2) w[2] = pj;
-      else w[3] = pj;
-      E[(size_t)r * bj + j] = ej;
-      Wpre[(size_t)r * bj + j] = wj;
     }
   }
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
     const int q = lane + 32 * u;
-    if (q < bj) W32[(size_t)r * k + i + q] = w[u];
+    if (q < bj) {
+      W32[(size_t)r * k + i + q] = w[u];
+      EW[(size_t)r * bj + q] = ew[u];
+    }
+  }
+}
+
+// Z (k x 2k row-major, as float2 pairs): Z[r][c] = {-L[r][c], D[c][r]}, so that
+// the lazy batch of a block is one product of K = 2 B_j: for row q after the
+// block, sum over the block's columns c of -L[q][c] E[.][c] + D[c][q] W_pre[.][c].
+// 32 x 32 tiles; D's tile goes through shared memory to be read transposed.
+__global__ void __launch_bounds__(256) build_z_kernel(const float* __restrict__ L, const float* __restrict__ D,
+                                                      int k, float2* __restrict__ Z) {
+  __shared__ float t[32][33];
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8
+  for (int y = ty; y < 32; y += 8) {   // t[c - c0][r - r0] = D[c][r]
+    const int c = c0 + y, r = r0 + tx;
+    t[y][tx] = (c < k && r < k) ? D[(size_t)c * k + r] : 0.f;
+  }
+  __syncthreads();
+  for (int y = ty; y < 32; y += 8) {
+    const int r = r0 + y, c = c0 + tx;
+    if (r < k && c < k) Z[(size_t)r * k + c] = make_float2(-L[(size_t)r * k + c], t[tx][y]);
   }
 }
 
@@ -620,12 +673,16 @@ struct duo_calib {
   void* allocs[32];
   int nalloc;
   // column sweep scratch, grown on demand: W32 (n x k fp32), keep (n x k),
-  // E and W_pre (n x 128 fp32 each)
-  float *sw_W32, *sw_E, *sw_Wpre;
+  // {E, W_pre} pairs (n x 128 float2); Z (k x k float2) is rebuilt after
+  // every precompute (z_ok = 0)
+  float* sw_W32;
+  float2* sw_EW;
+  float2* sw_Z;
+  int z_ok;
   uint8_t* sw_keep;
   uint32_t *sw_keys, *sw_ctacnt;
   int64_t sw_rows;
-  uint32_t* sel_hist;             // 65536 bins, zero between passes
+  uint32_t* sel_hist;             // 2048 bins, zero between passes
   duo::calib::SelState* sel_state;
 };
 
@@ -657,8 +714,8 @@ void release(duo_calib* h) {
   if (h->solver) cusolverDnDestroy(h->solver);
   for (int i = 0; i < h->nalloc; ++i) cudaFree(h->allocs[i]);
   cudaFree(h->sw_W32);
-  cudaFree(h->sw_E);
-  cudaFree(h->sw_Wpre);
+  cudaFree(h->sw_EW);
+  cudaFree(h->sw_Z);
   cudaFree(h->sw_keep);
   cudaFree(h->sw_keys);
   cudaFree(h->sw_ctacnt);
@@ -764,6 +821,7 @@ int duo_calib_precompute(duo_calib* h, const void* X_fp16_dev, int64_t keep, flo
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const int k = (int)h->k, m = (int)h->m;
   const uint16_t* X = static_cast<const uint16_t*>(X_fp16_dev);
+  h->z_ok = 0;   // the sweep's Z follows this precompute's L and D
   // 1. X_hat and dX, one token per CTA
   const size_t tsm = tok_xs_bytes(k) + sizeof(duo::SelShared);
   cudaError_t e = cudaFuncSetAttribute(token_sparsify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -928,19 +986,18 @@ int duo_calib_prune(duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw
     e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return map_cuda(e);
     cudaFree(h->sw_W32);
-    cudaFree(h->sw_E);
-    cudaFree(h->sw_Wpre);
+    cudaFree(h->sw_EW);
     cudaFree(h->sw_keep);
     cudaFree(h->sw_keys);
     cudaFree(h->sw_ctacnt);
-    h->sw_W32 = h->sw_E = h->sw_Wpre = nullptr;
+    h->sw_W32 = nullptr;
+    h->sw_EW = nullptr;
     h->sw_keep = nullptr;
     h->sw_keys = h->sw_ctacnt = nullptr;
     h->sw_rows = 0;
     const size_t nk = (size_t)n * k;
     e = cudaMalloc(&h->sw_W32, nk * sizeof(float));
-    if (e == cudaSuccess) e = cudaMalloc(&h->sw_E, (size_t)n * 128 * sizeof(float));
-    if (e == cudaSuccess) e = cudaMalloc(&h->sw_Wpre, (size_t)n * 128 * sizeof(float));
+    if (e == cudaSuccess) e = cudaMalloc(&h->sw_EW, (size_t)n * 128 * sizeof(float2));
     if (e == cudaSuccess) e = cudaMalloc(&h->sw_keep, nk);
     if (e == cudaSuccess) e = cudaMalloc(&h->sw_keys, (size_t)n * 128 * sizeof(uint32_t));
     if (e == cudaSuccess)
@@ -949,45 +1006,57 @@ int duo_calib_prune(duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw
     h->sw_rows = n;
   }
   float* W32 = h->sw_W32;
-  float* E = h->sw_E;
-  float* Wpre = h->sw_Wpre;
+  float2* EW = h->sw_EW;
+  if (h->sw_Z == nullptr) {
+    e = cudaMalloc(&h->sw_Z, (size_t)k * k * sizeof(float2));
+    if (e != cudaSuccess) return map_cuda(e);
+    h->z_ok = 0;
+  }
+  if (!h->z_ok) {
+    const dim3 gz((k + 31) / 32, (k + 31) / 32);
+    build_z_kernel<<<gz, 256, 0, st>>>(h->L, h->D, k, h->sw_Z);
+    h->z_ok = 1;
+  }
   uint8_t* keepP = h->sw_keep;
   const dim3 gk((k + 255) / 256, (unsigned)n);
   load_permuted_kernel<<<gk, 256, 0, st>>>(static_cast<const uint16_t*>(W_fp16_dev), ldw, k, h->perm, W32);
-  const size_t ssm = (size_t)block * block * sizeof(float2);
-  e = cudaFuncSetAttribute(block_sweep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssm);
+  e = cudaFuncSetAttribute(block_sweep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SWEEP_SMEM);
   if (e != cudaSuccess) return map_cuda(e);
   if (cublasSetStream(h->blas, st) != CUBLAS_STATUS_SUCCESS) return DUO_ECUDA;
-  const float one = 1.f, minus_one = -1.f;
+  const float one = 1.f;
+  // rows (warps) per CTA of the in-block sweep: one CTA per SM, waves of 152
+  const int64_t waves = (n + (int64_t)152 * SWEEP_ROWS - 1) / ((int64_t)152 * SWEEP_ROWS);
+  const int rpc = (int)((n + 152 * waves - 1) / (152 * waves));
   for (int i = 0; i < k; i += block) {
     const int bj = k - i < block ? k - i : block;
     const int64_t cnt = (int64_t)n * bj * pw_pct / 100;
     const int64_t N = (int64_t)n * bj;
     const unsigned nb = (unsigned)((N + SELM_PER_CTA - 1) / SELM_PER_CTA);
-    sel_keys_kernel<<<nb, SELM_THREADS, 0, st>>>(W32, k, i, bj, N, h->col, h->sw_keys, h->sel_hist);
+    const unsigned nh = nb < 2u * 152u ? nb : 2u * 152u;   // histogram CTAs, grid-strided
+    sel_keys_kernel<<<nh, SELM_THREADS, 0, st>>>(W32, (int)n, k, i, bj, h->col, h->sw_keys, h->sel_hist);
     sel_pick_kernel<<<1, 1024, 0, st>>>(h->sel_hist, h->sel_state, 0, (uint32_t)cnt);
-    sel_low_hist_kernel<<<nb, SELM_THREADS, 0, st>>>(h->sw_keys, N, h->sel_state, h->sel_hist);
+    sel_hist_kernel<<<nh, SELM_THREADS, 0, st>>>(h->sw_keys, N, h->sel_state, 1, h->sel_hist);
     sel_pick_kernel<<<1, 1024, 0, st>>>(h->sel_hist, h->sel_state, 1, (uint32_t)cnt);
+    sel_hist_kernel<<<nh, SELM_THREADS, 0, st>>>(h->sw_keys, N, h->sel_state, 2, h->sel_hist);
+    sel_pick_kernel<<<1, 1024, 0, st>>>(h->sel_hist, h->sel_state, 2, (uint32_t)cnt);
     sel_tie_count_kernel<<<nb, SELM_THREADS, 0, st>>>(h->sw_keys, N, h->sel_state, h->sw_ctacnt);
     sel_tie_scan_kernel<<<1, 1024, 0, st>>>(h->sw_ctacnt, (int)nb);
     sel_mask_kernel<<<nb, SELM_THREADS, 0, st>>>(h->sw_keys, N, k, i, bj, h->sel_state, h->sw_ctacnt,
                                                  cnt == 0 ? 1 : 0, keepP);
-    block_sweep_kernel<<<(unsigned)((n + SWEEP_ROWS - 1) / SWEEP_ROWS), SWEEP_ROWS * 32, ssm, st>>>(
-        W32, (int)n, k, i, bj, h->L, h->D, keepP, E, Wpre);
+    block_sweep_kernel<<<(unsigned)((n + rpc - 1) / rpc), (unsigned)rpc * 32, SWEEP_SMEM, st>>>(
+        W32, (int)n, k, i, bj, h->sw_Z, h->L, keepP, EW);
     e = cudaGetLastError();
     if (e != cudaSuccess) return map_cuda(e);
     const int nt = k - i - bj;   // trailing columns
     if (nt > 0) {
-      // Lazy batch: W_T -= E L_T,blk^T - W_pre D_blk,T.  Row-major buffers are
-      // column-major transposes: W_T^T (nt x n, ld k) += -(L^T)[blk, T]^T E^T
-      // + (D^T)[T, blk] W_pre^T.
-      int rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_T, CUBLAS_OP_N, nt, (int)n, bj, &minus_one,
-                                     h->L + i + (size_t)(i + bj) * k, CUDA_R_32F, k, E, CUDA_R_32F, bj, &one,
-                                     W32 + i + bj, CUDA_R_32F, k, kL_COMPUTE, CUBLAS_GEMM_DEFAULT));
-      if (rc != DUO_OK) return rc;
-      rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_N, CUBLAS_OP_N, nt, (int)n, bj, &one,
-                                 h->D + (i + bj) + (size_t)i * k, CUDA_R_32F, k, Wpre, CUDA_R_32F, bj, &one,
-                                 W32 + i + bj, CUDA_R_32F, k, kL_COMPUTE, CUBLAS_GEMM_DEFAULT));
+      // Lazy batch: W_T -= E L_T,blk^T - W_pre D_blk,T as one product of
+      // K = 2 B_j over the pairs: row-major buffers are column-major
+      // transposes, W_T^T (nt x n, ld k) += Z[T, blk]^T-view (nt x 2bj, read
+      // with OP_T from ld 2k) times {E, W_pre}^T (2bj x n, ld 2bj).
+      const float* Zb = reinterpret_cast<const float*>(h->sw_Z) + (size_t)(i + bj) * 2 * k + 2 * (size_t)i;
+      int rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_T, CUBLAS_OP_N, nt, (int)n, 2 * bj, &one, Zb,
+                                     CUDA_R_32F, 2 * k, EW, CUDA_R_32F, 2 * bj, &one, W32 + i + bj,
+                                     CUDA_R_32F, k, kL_COMPUTE, CUBLAS_GEMM_DEFAULT));
       if (rc != DUO_OK) return rc;
     }
   }
