@@ -617,9 +617,10 @@ def run_e2e(duo, shape, layers, args, breq_mean):
     """End to end through the public API: every step copies that layer's
     inputs from pinned host memory to the device, runs the four stage calls
     and copies every output back.  Measured two ways: with duo.StepGraph
-    (the step captured once, one replay call per step, one copy each way:
-    the serving call) as the reported value, and with the individual calls
-    and per-tensor copies issued eagerly from Python each step."""
+    (the step captured once, one replay call per step, one SM-kernel copy
+    each way: the serving call) as the reported value, and with the
+    individual calls and per-tensor copy-engine copies issued eagerly from
+    Python each step."""
     L = len(layers)
     hx = [{s: layers[l]["x"][s].cpu().pin_memory() for s in STAGE_SRC} for l in range(L)]
     hy = [{p: torch.empty(shape.O(p), dtype=torch.float32).pin_memory() for p in layers[l]["y"]}
@@ -661,8 +662,10 @@ def run_e2e(duo, shape, layers, args, breq_mean):
     del plans
     return {"value": breq_mean * n / t_graph / 1e9, "unit": "GB/s", "us_per_layer": t_graph / n * 1e6,
             "h2d_bytes_per_step": h2d_graph, "d2h_bytes_per_step": d2h_graph, "steps": n,
-            "api": "duo.StepGraph: one H2D copy of the step's inputs, the 4 stage calls, one D2H copy "
-                   "of all outputs, replayed as one graph per step",
+            "api": "duo.StepGraph: the step's inputs copied in from pinned host memory and all "
+                   "outputs copied back by the library's SM copy kernel (duo_copy), the 4 stage "
+                   "calls between, replayed as one graph per step",
+            "gpu_launches_per_step": 2 + len(STAGES),
             "eager_calls": {"value": breq_mean * n / t_eager / 1e9, "us_per_layer": t_eager / n * 1e6,
                             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}}
 

@@ -271,6 +271,23 @@ int duo_pack_cmb_noalloc(const void* W_fp16_dev, int64_t out, int64_t in, int64_
                          uint32_t* off_dev, void* data_dev, int64_t data_capacity,
                          int64_t* data_bytes, void* stream);
 
+/*
+ * duo_copy -- copies `bytes` bytes from src to dst with a kernel on the SMs
+ * (asynchronous on `stream`, a cudaStream_t passed as void*).  Each pointer
+ * is device memory of the current device, managed memory, or page-locked host
+ * memory mapped into the device's address space (cudaHostAlloc /
+ * cudaHostRegister memory on a system with unified addressing); the caller
+ * owns both, and both ranges must lie inside their allocations and not
+ * overlap.  Any alignment; 16-byte aligned ends copy in 16-byte words.  Not a
+ * step of the method: it moves a decode step's inputs in and outputs out
+ * without a copy-engine node, the cheaper choice inside a captured step.
+ * The kernel first waits for the stream's previous kernel to complete.
+ * Errors: DUO_EINVAL (NULL, bytes < 0, a pointer the device cannot reach:
+ * unregistered host memory, another device's memory), DUO_ECUDA (no device,
+ * launch).  bytes = 0 returns DUO_OK at once (NULL pointers allowed).
+ */
+int duo_copy(void* dst, const void* src, int64_t bytes, void* stream);
+
 /* Synchronises `stream`, returns and clears the device status word:
  * DUO_OK; DUO_ETIMEOUT if a bounded device wait ran out since the last
  * call; DUO_EFORMAT if a kernel met a record size or channel id outside the

@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT = os.path.join(PKG, "libduo.so")
 BUILD_DIR = os.path.join(PKG, "_build")
-SOURCES = ("kernels.cu", "api.cu", "noalloc.cu", "calib.cu")
+SOURCES = ("kernels.cu", "api.cu", "noalloc.cu", "calib.cu", "copy.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -60,6 +60,7 @@ def load_library(path: str | None = None):
     lib.duo_packed_export.argtypes = [vp, i32, vp, i64]
     lib.duo_pack_cmb_noalloc.argtypes = [vp, i64, i64, i64, vp, vp, i64, ctypes.POINTER(i64), vp]
     lib.duo_device_status.argtypes = [vp]
+    lib.duo_copy.argtypes = [vp, vp, i64, vp]
     lib.duo_calib_create.argtypes = [i64, i64, vp, ctypes.POINTER(vp)]
     lib.duo_calib_precompute.argtypes = [vp, vp, i64, ctypes.c_float, i32, vp]
     lib.duo_calib_status.argtypes = [vp, vp]
@@ -73,7 +74,7 @@ def load_library(path: str | None = None):
                  "duo_packed_query", "duo_packed_export", "duo_device_status", "duo_abi_version",
                  "duo_pack_cmb_noalloc", "duo_sparsify_threshold", "duo_spmspv_threshold",
                  "duo_calib_create", "duo_calib_precompute", "duo_calib_status", "duo_calib_export",
-                 "duo_calib_score", "duo_calib_free", "duo_calib_prune"):
+                 "duo_calib_score", "duo_calib_free", "duo_calib_prune", "duo_copy"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -244,6 +245,17 @@ def duo_device_status(stream=None) -> int:
     return load_library().duo_device_status(_stream_ptr(stream))
 
 
+def duo_copy(dst: torch.Tensor, src: torch.Tensor, stream=None):
+    """dst <- src (same byte size, contiguous) by the library's SM copy
+    kernel; either side may be a CUDA tensor or a pinned host tensor."""
+    if not (dst.is_contiguous() and src.is_contiguous()):
+        raise ValueError("duo_copy needs contiguous tensors")
+    n = dst.numel() * dst.element_size()
+    if src.numel() * src.element_size() != n:
+        raise ValueError("duo_copy: sizes differ")
+    _check(load_library().duo_copy(dst.data_ptr(), src.data_ptr(), n, _stream_ptr(stream)), "duo_copy")
+
+
 def packed_bytes(h: Packed):
     """Copies a handle's index / aux / data buffers to host numpy uint8
     arrays through duo_packed_export (byte-level parity checks, saving)."""
@@ -357,7 +369,8 @@ class StepGraph:
     """A decode step of several dual-sparse products, captured once as a
     CUDA graph and replayed with one call: one host -> device copy of all the
     step's inputs, the products back to back, one device -> host copy of all
-    outputs.
+    outputs.  The two copies are the library's SM copy kernel (duo_copy) on
+    the pinned buffers, not copy-engine nodes (about 4 us less per step).
 
     ``stages`` is a list of dicts: ``h`` (a Packed, or a list of up to 4
     sharing one input) and ``k`` (kept channels).  The object owns one pinned
@@ -402,7 +415,7 @@ class StepGraph:
         return self._yh[off:off + O]
 
     def _enqueue(self):
-        self._xd.copy_(self._xh, non_blocking=True)
+        duo_copy(self._xd, self._xh)
         for hs, k, xo, I, yo in self._stages:
             x = self._xd[xo:xo + I]
             ys = [self._yd[o:o + O] for o, O in yo]
@@ -410,7 +423,7 @@ class StepGraph:
                 duo_spmspv(hs[0], x, k, y=ys[0])
             else:
                 duo_spmspv_multi(hs, x, k, ys=ys)
-        self._yh.copy_(self._yd, non_blocking=True)
+        duo_copy(self._yh, self._yd)
 
     def run(self):
         self.graph.replay()

@@ -152,3 +152,18 @@ def test_calib_argument_validation(lib):
     assert lib.duo_calib_prune(None, FAKE, 4, 8, 50, 128, FAKE, None, None) == EINVAL
     assert lib.duo_calib_free(FAKE) == EINVAL
     assert lib.duo_calib_free(None) == 0
+
+
+def test_copy_argument_validation(lib):
+    """duo_copy rejects NULL ends and negative sizes before touching the
+    GPU, accepts an empty copy at once; an unknown address is refused (EINVAL where CUDA can classify it,
+    ECUDA where no device is present), never copied."""
+    vp, i64 = ctypes.c_void_p, ctypes.c_int64
+    lib.duo_copy.argtypes = [vp, vp, i64, vp]
+    EINVAL, ECUDA = -1, -3
+    assert lib.duo_copy(None, FAKE, 16, None) == EINVAL
+    assert lib.duo_copy(FAKE, None, 16, None) == EINVAL
+    assert lib.duo_copy(FAKE, FAKE, -1, None) == EINVAL
+    assert lib.duo_copy(None, None, 0, None) == 0
+    assert lib.duo_copy(FAKE, FAKE, 16, None) in (EINVAL, ECUDA)
+

@@ -416,3 +416,43 @@ def test_step_graph_copies_and_products(duo):
             assert np.all(err <= orc.tolerance_rows(W, x, K)), trial
     for h in hs + [h2]:
         h.free()
+
+
+@pytest.mark.parametrize("nbytes,off", [(0, 0), (1, 0), (15, 1), (16, 0), (17, 3), (12293, 0), (12293, 2),
+                                        (1 << 20, 0)])
+def test_copy_kernel_bytes(duo, nbytes, off):
+    """duo_copy moves exactly the bytes asked for, device <-> pinned host and
+    device -> device, aligned (16-byte words) and misaligned (byte path),
+    and writes nothing past the range."""
+    d = duo
+    rng = np.random.default_rng(nbytes + off)
+    src = torch.from_numpy(rng.integers(0, 256, size=nbytes + 32, dtype=np.uint8)).pin_memory()
+    dev = torch.full((nbytes + 32,), 0xA5, dtype=torch.uint8, device="cuda")
+    back = torch.full((nbytes + 32,), 0x5A, dtype=torch.uint8).pin_memory()
+    dev2 = torch.full((nbytes + 32,), 0x3C, dtype=torch.uint8, device="cuda")
+    d.duo_copy(dev[off:off + nbytes], src[off:off + nbytes])
+    d.duo_copy(dev2[off:off + nbytes], dev[off:off + nbytes])
+    d.duo_copy(back[off:off + nbytes], dev2[off:off + nbytes])
+    torch.cuda.synchronize()
+    s, b = src.numpy(), back.numpy()
+    assert np.array_equal(b[off:off + nbytes], s[off:off + nbytes])
+    assert np.all(b[:off] == 0x5A) and np.all(b[off + nbytes:] == 0x5A)
+    dv = dev.cpu().numpy()
+    assert np.all(dv[:off] == 0xA5) and np.all(dv[off + nbytes:] == 0xA5)
+    assert d.duo_device_status() == 0
+
+
+def test_copy_kernel_rejects_pageable_host_memory(duo):
+    """Plain (unpinned) host memory is refused on the host with EINVAL; the
+    stream stays usable."""
+    d = duo
+    pageable = torch.zeros(64, dtype=torch.uint8)
+    dev = torch.zeros(64, dtype=torch.uint8, device="cuda")
+    with pytest.raises(d.DuoError):
+        d.duo_copy(dev, pageable)
+    with pytest.raises(d.DuoError):
+        d.duo_copy(pageable, dev)
+    d.duo_copy(dev, torch.ones(64, dtype=torch.uint8).pin_memory())
+    torch.cuda.synchronize()
+    assert int(dev.sum()) == 64
+
