@@ -57,6 +57,8 @@ def parse():
                     help="small case for ncu: one 7B layer's four stages once per format (fp16, 8-bit, 4-bit)")
     ap.add_argument("--profile-calib", action="store_true",
                     help="small case for ncu: `--steps` calibration precomputes of a 4096-channel layer")
+    ap.add_argument("--profile-sweep", action="store_true",
+                    help="small case for ncu: one precompute, then `--steps` column sweeps of a 4096 x 4096 weight")
     ap.add_argument("--stack", default=None,
                     choices=("llama2-7b-layer", "llama3-8b-stack", "llama2-13b-stack", "llama2-70b-stack"),
                     help="per-token time over every layer of a stack workload (one CUDA graph per token)")
@@ -737,8 +739,10 @@ def run_profile_coded(args):
 
 
 def run_profile_calib(args):
-    """Calibration precompute for profiler captures: one 4096-channel layer
-    from 2048 tokens, one warm-up and `--steps` precomputes, no graphs."""
+    """Calibration for profiler captures: one 4096-channel layer from 2048
+    tokens, one warm-up and `--steps` precomputes, no graphs; with
+    --profile-sweep one precompute and then `--steps` column sweeps of a
+    4096 x 4096 weight (B = 128, 50% per block)."""
     torch.cuda.set_device(0)
     import __graft_entry__
     __graft_entry__.build()
@@ -749,9 +753,15 @@ def run_profile_calib(args):
     u = torch.rand(m, k, generator=g, device="cuda", dtype=torch.float32) - 0.5
     X = (-torch.sign(u) * torch.log1p(-2 * u.abs())).to(torch.float16)
     c = duo.Calib(k, m)
-    for _ in range(1 + args.steps):
+    for _ in range(1 if args.profile_sweep else 1 + args.steps):
         c.precompute(X, k // 2)
     assert c.status() == duo.DUO_OK
+    if args.profile_sweep:   # Algorithm 1's column sweep, B = 128, 50% per block
+        W = (torch.randn(k, k, generator=g, device="cuda") * 0.02).to(torch.float16)
+        for _ in range(args.steps):
+            c.prune(W, 50, 128)
+        torch.cuda.synchronize()
+        assert c.status() == duo.DUO_OK
     c.free()
     print("profile workload done", flush=True)
 
@@ -823,7 +833,7 @@ def main():
     args = parse()
     if args.profile:
         run_profile(args)
-    elif args.profile_calib:
+    elif args.profile_calib or args.profile_sweep:
         run_profile_calib(args)
     elif args.profile_coded:
         run_profile_coded(args)
