@@ -155,6 +155,37 @@ def k_of(I, px):
     return (I * (100 - px)) // 100
 
 
+def side_bytes_layer(duo, shape, layer, px):
+    """Companions of the required bytes of one layer step: the kept
+    non-zero values alone (2 sum nnz_j over kept j: the weights loaded, the
+    quantity the paper counts), and the worst case of the required-bytes
+    formula, with the k densest channels of each stage selected instead of
+    the ones x picks; then the values of both as fractions of the dense
+    weights (Fig. 3's loaded fraction and its worst case, App. B.3)."""
+    vals = worst = wvals = dense = 0.0
+    for st, src in zip(STAGES, STAGE_SRC):
+        I = shape.I(st[0])
+        k = k_of(I, px)
+        if k == 0:
+            worst += 2.0 * I
+            continue
+        idx, _ = duo.duo_sparsify(layer["x"][src], k)
+        K = idx.to(torch.int64) & 0xFFFF
+        tot = sum(layer["nnz"][p] for p in st)            # per channel, over the stage's products
+        dense_k = torch.topk(tot, k).indices
+        for p in st:
+            O = shape.O(p)
+            vals += float(layer["nnz"][p][K].sum().item()) * 2.0
+            wv = float(layer["nnz"][p][dense_k].sum().item()) * 2.0
+            wvals += wv
+            worst += wv + k * O / 8.0 + 4.0 * O
+        worst += 2.0 * I + 4.0 * k
+    for st in STAGES:
+        for p in st:
+            dense += 2.0 * shape.O(p) * shape.I(p)
+    return vals, worst, vals / dense, wvals / dense
+
+
 def required_bytes_layer(duo, shape, layer, px):
     """Format-neutral required bytes of one layer step, with the kept sets
     taken from the library's own (parity-tested) sparsifier."""
@@ -376,6 +407,7 @@ def run_ours(args):
     shape, layers = make_layers(duo, synth, L, dev, args.px)
     breq_layers = [required_bytes_layer(duo, shape, lay, args.px) for lay in layers]
     breq_mean = float(np.mean([b for b, _ in breq_layers]))
+    side = np.mean(np.array([side_bytes_layer(duo, shape, lay, args.px) for lay in layers]), axis=0)
     stage_b = np.mean(np.array([ps for _, ps in breq_layers]), axis=0)
 
     g = capture_rotation(duo, shape, layers, args.px)
@@ -454,7 +486,12 @@ def run_ours(args):
                        "pw": 0.5, "prune": "magnitude, exact count per 128-channel block",
                        "px": args.px, "format": "bitmask (CMB)", "layers_rotated": L,
                        "l2": f"inputs larger than L2: {L} distinct packed layers rotated",
-                       "required_MB_per_layer": breq_mean / 1e6, "parallelism": "replicas" if world > 1 else "1gpu"},
+                       "required_MB_per_layer": breq_mean / 1e6,
+                       "vals_only_MB_per_layer": float(side[0]) / 1e6,
+                       "worst_case_required_MB_per_layer": float(side[1]) / 1e6,
+                       "loaded_weight_fraction": float(side[2]),
+                       "worst_case_loaded_weight_fraction": float(side[3]),
+                       "parallelism": "replicas" if world > 1 else "1gpu"},
             "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": e2e,

@@ -311,14 +311,24 @@ __device__ __forceinline__ int select_bit(uint32_t m, int r) {
   return pos;
 }
 
-// Block-cooperative copy of x (fp16 bits) into shared memory.
+// Block-cooperative copy of x (fp16 bits) into shared memory.  Up to four
+// 16-byte loads per thread are issued before the first store, so a thread
+// waits for one memory round trip per 4 blocks of the input, not per block.
 __device__ inline void load_x_to_smem(uint16_t* xs, const uint16_t* x, int I) {
   const int tid = threadIdx.x, nt = blockDim.x;
   if ((reinterpret_cast<uintptr_t>(x) & 15u) == 0) {
     const int nvec = I >> 3;
     const uint4* xv = reinterpret_cast<const uint4*>(x);
     uint4* sv = reinterpret_cast<uint4*>(xs);
-    for (int i = tid; i < nvec; i += nt) sv[i] = __ldg(xv + i);
+    for (int i0 = tid; i0 < nvec; i0 += 4 * nt) {
+      uint4 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (i0 + u * nt < nvec) v[u] = __ldg(xv + i0 + u * nt);
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (i0 + u * nt < nvec) sv[i0 + u * nt] = v[u];
+    }
     for (int i = (nvec << 3) + tid; i < I; i += nt) xs[i] = x[i];
   } else {
     for (int i = tid; i < I; i += nt) xs[i] = x[i];

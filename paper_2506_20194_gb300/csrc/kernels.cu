@@ -728,13 +728,14 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   if (MODE == CMB_TOPK) select_clear(sel);
   // Inputs, y and the grid barrier words may be the previous kernel's.
   griddep_wait();
-  if (FUSED) load_x_to_smem(xs, a.x, a.I);
   // Generation of the grid barrier before this CTA arrives on it (read here,
-  // before any of this CTA's warps can arrive).
+  // before any of this CTA's warps can arrive; issued ahead of the x loads
+  // so that the two round trips overlap).
   unsigned int gen0 = 0;
   if (tid == 0) {
     gen0 = ld_relaxed_gpu(a.bar + 1);
   }
+  if (FUSED) load_x_to_smem(xs, a.x, a.I);
   uint32_t u0, u1;   // this CTA's items (32-bit: the launcher keeps counts < 2^31)
   int r0 = 0;        // kept rank of its first item
   int pr = 0, sr = 0, c0 = 0, c1 = 0;   // fused modes: run (product, segment), channel range
