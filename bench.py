@@ -36,8 +36,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch of
 # the fused kernel from one ncu capture, valid only for the kernel source it
 # was taken on (sha256 of kernels.cu + duo_device.cuh, first 16 hex digits).
-TRAFFIC = {"sha": "3acf777159afa7db",
-           "per_launch_bytes": [29105664.0, 9753088.0, 51889152.0, 26097920.0]}
+TRAFFIC = {"sha": "08b3b6942fafab2b",
+           "per_launch_bytes": [29107456.0, 9751808.0, 51892992.0, 26098432.0]}
 
 
 def parse():
