@@ -8,7 +8,8 @@ seeded layers rotate so that every step streams weights that are not in L2.
 
 Printed metric: effective HBM GB/s on the required bytes (the kept channels'
 fp16 non-zeros, one mask bit per kept position, x, kept ids/values and y),
-plus microseconds per layer.  See the design doc for the byte model.
+plus microseconds per layer.  Padding, offset tables and index bytes are not
+required bytes; the DRAM counters of a profile show them.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 """
@@ -19,6 +20,7 @@ import json
 import math
 import os
 import subprocess
+import tempfile
 import sys
 import time
 
@@ -97,7 +99,8 @@ class ClockSampler:
     def __init__(self, index: int):
         self.index = index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+        out = os.environ.get("DUO_CLOCKS_DIR") or tempfile.gettempdir()
+        self.path = os.path.join(out, f"clocks_rank{index}.csv")
 
     def start(self):
         try:

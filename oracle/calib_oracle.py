@@ -17,7 +17,7 @@ magnitude (§3, "Activation Sparsity"); X_tilde is the dense input.
     S[:, p] = W[:, p]^2 (1 / L_pp^2 + a_p - b_p + 2 c_p)      (the efficient score)
 
 Readings (the paper's calibration settings, App. B.1, plus points it leaves
-open; each is listed in DESIGN.md):
+open):
   * X_hat keeps, per token column, the keep = floor(k (100 - pct) / 100)
     channels of largest |x| (ties to the lower channel index), as the decode
     sparsifier does;

@@ -15,7 +15,7 @@ and only the weight columns of the surviving channels are fetched (§4.1).
 Weight sparsity is unstructured: a pruned weight is stored as zero (§3, mask
 m^w), and each kept column is stored compressed (§4.1).
 
-Readings taken where the paper is silent (each is listed in the design doc):
+Readings taken where the paper is silent:
   * the number of kept channels is k = floor(I * (100 - pct) / 100) for an
     integer activation-sparsity percentage pct;
   * the kept set is the k channels of largest |x_j|; ties between equal
