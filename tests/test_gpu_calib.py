@@ -130,6 +130,26 @@ def test_sweep_matches_oracle(duo, n, k, m, keep, pw, block):
     _close("W", out, Wref, TOL_FACTOR)
 
 
+@pytest.mark.parametrize("n,k,m,keep,pw,block", [(40, 100, 200, 50, 0, 32), (40, 100, 200, 50, 100, 32),
+                                                  (24, 70, 150, 35, 50, 1), (1, 160, 300, 80, 50, 64),
+                                                  (17, 129, 260, 64, 33, 128)])
+def test_sweep_degenerate_cases(duo, n, k, m, keep, pw, block):
+    """Edge cases of the sweep against the fp64 oracle: nothing pruned
+    (every entry kept; the weights still move by the activation-sparsity
+    term W_j D_jq), everything pruned (all zero), blocks of one column, a
+    single row, and a last block of one column (k = 129, B = 128)."""
+    W, pre, out, kmask = _sweep(duo, n, k, m, keep, pw, block, seed=n * 7 + k)
+    Wref, mref = orc.oracle_calib_prune_blocked(W, pre, pw, block)
+    assert np.array_equal(kmask, mref)
+    assert np.all(out[~kmask] == 0)
+    if pw == 0:
+        assert kmask.all()
+    if pw == 100:
+        assert not kmask.any() and np.all(out == 0)
+    else:
+        _close("W", out, Wref, TOL_FACTOR)
+
+
 def test_sweep_full_size_layer(duo):
     """4096 x 4096 weight, 2048 tokens, B = 128, 50%: exact counts per block,
     pruned entries zero; against the fp64 oracle, the first block's mask is
