@@ -328,12 +328,13 @@ __device__ __forceinline__ uint32_t score_key(float s) {
 // global one over the non-empty bins) followed by a one-CTA pick of the
 // digit, give the cnt-th smallest key T and `want`, the number of elements
 // equal to T to prune; per-CTA tie counts and their scan then give every tie
-// its rank in flat order.  Elements are split into contiguous flat ranges of
-// SELM_PER_CTA, SELM_PER_THREAD consecutive ones per thread.
+// its rank in flat order.  The histogram kernels are grid-strided; the tie
+// and mask kernels split the elements into contiguous flat ranges of
+// SELM_PER_CTA per CTA, SELM_PER_THREAD consecutive ones per thread.
 constexpr int SELM_THREADS = 256;
 constexpr int SELM_PER_THREAD = 8;
 constexpr int SELM_PER_CTA = SELM_THREADS * SELM_PER_THREAD;
-constexpr int SEL_BINS16 = 2048;   // the largest digit (11 bits)
+constexpr int SEL_DIGIT_BINS = 2048;   // the largest digit (11 bits)
 
 struct SelState {
   uint32_t prefix;   // T once all passes have run
@@ -350,8 +351,8 @@ __global__ void __launch_bounds__(SELM_THREADS) sel_keys_kernel(const float* __r
                                                                 const float* __restrict__ col,
                                                                 uint32_t* __restrict__ keys,
                                                                 uint32_t* __restrict__ hist) {
-  __shared__ uint32_t h[SEL_BINS16];
-  for (int b = threadIdx.x; b < SEL_BINS16; b += SELM_THREADS) h[b] = 0u;
+  __shared__ uint32_t h[SEL_DIGIT_BINS];
+  for (int b = threadIdx.x; b < SEL_DIGIT_BINS; b += SELM_THREADS) h[b] = 0u;
   __syncthreads();
   const int64_t N = (int64_t)n * bj;
   const int stride = (int)gridDim.x * SELM_THREADS;
@@ -372,7 +373,7 @@ __global__ void __launch_bounds__(SELM_THREADS) sel_keys_kernel(const float* __r
     }
   }
   __syncthreads();
-  for (int b = threadIdx.x; b < SEL_BINS16; b += SELM_THREADS)
+  for (int b = threadIdx.x; b < SEL_DIGIT_BINS; b += SELM_THREADS)
     if (h[b]) atomicAdd(&hist[b], h[b]);
 }
 
@@ -380,8 +381,8 @@ __global__ void __launch_bounds__(SELM_THREADS) sel_keys_kernel(const float* __r
 __global__ void __launch_bounds__(SELM_THREADS) sel_hist_kernel(const uint32_t* __restrict__ keys, int64_t N,
                                                                 const SelState* __restrict__ st, int pass,
                                                                 uint32_t* __restrict__ hist) {
-  __shared__ uint32_t h[SEL_BINS16];
-  for (int b = threadIdx.x; b < SEL_BINS16; b += SELM_THREADS) h[b] = 0u;
+  __shared__ uint32_t h[SEL_DIGIT_BINS];
+  for (int b = threadIdx.x; b < SEL_DIGIT_BINS; b += SELM_THREADS) h[b] = 0u;
   __syncthreads();
   const int sh = sel_shift(pass);
   const uint32_t hi = st->prefix >> (sh + (pass == 1 ? 11 : 10));
@@ -391,7 +392,7 @@ __global__ void __launch_bounds__(SELM_THREADS) sel_hist_kernel(const uint32_t* 
     if ((key >> (sh + (pass == 1 ? 11 : 10))) == hi) atomicAdd(&h[(key >> sh) & dmask], 1u);
   }
   __syncthreads();
-  for (int b = threadIdx.x; b < SEL_BINS16; b += SELM_THREADS)
+  for (int b = threadIdx.x; b < SEL_DIGIT_BINS; b += SELM_THREADS)
     if (h[b]) atomicAdd(&hist[b], h[b]);
 }
 
@@ -682,7 +683,7 @@ struct duo_calib {
   uint8_t* sw_keep;
   uint32_t *sw_keys, *sw_ctacnt;
   int64_t sw_rows;
-  uint32_t* sel_hist;             // 2048 bins, zero between passes
+  uint32_t* sel_hist;             // SEL_DIGIT_BINS counters, zero between passes
   duo::calib::SelState* sel_state;
 };
 
@@ -776,9 +777,9 @@ int duo_calib_create(int64_t k, int64_t m, void* stream, duo_calib** out) {
   if (e == cudaSuccess) e = alloc(h, &h->key_lo, (size_t)k);
   if (e == cudaSuccess) e = alloc(h, &h->perm, (size_t)k);
   if (e == cudaSuccess) e = alloc(h, &h->info, 2);
-  if (e == cudaSuccess) e = alloc(h, &h->sel_hist, (size_t)duo::calib::SEL_BINS16);
+  if (e == cudaSuccess) e = alloc(h, &h->sel_hist, (size_t)duo::calib::SEL_DIGIT_BINS);
   if (e == cudaSuccess) e = alloc(h, &h->sel_state, 1);
-  if (e == cudaSuccess) e = cudaMemsetAsync(h->sel_hist, 0, sizeof(uint32_t) * duo::calib::SEL_BINS16, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->sel_hist, 0, sizeof(uint32_t) * duo::calib::SEL_DIGIT_BINS, st);
   if (e != cudaSuccess) return fail(map_cuda(e));
   // cuSOLVER workspace of the factorisation.
   size_t d1 = 0, h1 = 0;
