@@ -38,6 +38,15 @@ class _Info(ctypes.Structure):
                 ("data_dev", ctypes.c_void_p), ("data_bytes", ctypes.c_int64)]
 
 
+class _CalibInfo(ctypes.Structure):
+    """Mirror of duo_calib_info (include/duo_calib.h)."""
+    _fields_ = [("k", ctypes.c_int64), ("m", ctypes.c_int64),
+                ("perm_dev", ctypes.c_void_p), ("H_dev", ctypes.c_void_p), ("L_dev", ctypes.c_void_p),
+                ("Q_dev", ctypes.c_void_p), ("U_dev", ctypes.c_void_p), ("D_dev", ctypes.c_void_p),
+                ("a_dev", ctypes.c_void_p), ("b_dev", ctypes.c_void_p), ("c_dev", ctypes.c_void_p),
+                ("col_dev", ctypes.c_void_p)]
+
+
 def load_library(path: str | None = None):
     """Loads libduo.so (once).  Raises if it is missing: there is no
     CPU or PyTorch fallback for any entry point."""
@@ -64,17 +73,19 @@ def load_library(path: str | None = None):
     lib.duo_calib_create.argtypes = [i64, i64, vp, ctypes.POINTER(vp)]
     lib.duo_calib_precompute.argtypes = [vp, vp, i64, ctypes.c_float, i32, vp]
     lib.duo_calib_status.argtypes = [vp, vp]
+    lib.duo_calib_query.argtypes = [vp, ctypes.POINTER(_CalibInfo)]
     lib.duo_calib_export.argtypes = [vp, i32, vp, i64, vp]
     lib.duo_calib_score.argtypes = [vp, vp, i64, i64, vp, vp]
     lib.duo_calib_prune.argtypes = [vp, vp, i64, i64, i32, i32, vp, vp, vp]
     lib.duo_calib_free.argtypes = [vp]
     lib.duo_strerror.argtypes = [i32]
+    lib.duo_abi_version.argtypes = []
     lib.duo_strerror.restype = ctypes.c_char_p
     for name in ("duo_pack", "duo_sparsify", "duo_spmspv", "duo_spmspv_multi", "duo_free",
                  "duo_packed_query", "duo_packed_export", "duo_device_status", "duo_abi_version",
                  "duo_pack_cmb_noalloc", "duo_sparsify_threshold", "duo_spmspv_threshold",
                  "duo_calib_create", "duo_calib_precompute", "duo_calib_status", "duo_calib_export",
-                 "duo_calib_score", "duo_calib_free", "duo_calib_prune", "duo_copy"):
+                 "duo_calib_score", "duo_calib_free", "duo_calib_prune", "duo_copy", "duo_calib_query"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -322,6 +333,13 @@ class Calib:
 
     def status(self, stream=None) -> int:
         return load_library().duo_calib_status(self._h, _stream_ptr(stream))
+
+    def query(self) -> dict:
+        """duo_calib_query: k, m and the device addresses of the context's
+        buffers (owned by the context; valid until the next precompute)."""
+        info = _CalibInfo()
+        _check(load_library().duo_calib_query(self._h, ctypes.byref(info)), "duo_calib_query")
+        return {name: getattr(info, name) for name, _ in _CalibInfo._fields_}
 
     def get(self, name: str, stream=None) -> torch.Tensor:
         which, dt, nd = _CALIB_BUFS[name]

@@ -36,6 +36,26 @@ def test_header_declares_the_boundary():
         assert n in names
 
 
+def test_binding_types_every_declared_function(lib):
+    """The Python binding sets argument and result types for every function
+    include/*.h declares (no call goes through ctypes' int defaults)."""
+    for n in _declared_functions():
+        f = getattr(lib, n)
+        assert f.argtypes is not None, f"{n}: no argtypes in the binding"
+        assert f.restype is not None, f"{n}: no restype in the binding"
+
+
+def test_calib_info_mirror_matches_header():
+    """duo.py's ctypes mirror of duo_calib_info lists the header's fields in
+    the header's order."""
+    from paper_2506_20194_gb300 import duo
+    txt = open(os.path.join(ROOT, "include", "duo_calib.h")).read()
+    body = re.search(r"typedef struct duo_calib_info \{(.*?)\} duo_calib_info;", txt, flags=re.S).group(1)
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    fields = re.findall(r"(\w+)\s*[,;]", body)
+    assert fields == [name for name, _ in duo._CalibInfo._fields_]
+
+
 def test_library_exports_every_declared_symbol(lib):
     for n in _declared_functions():
         assert hasattr(lib, n), f"{n} declared in include/ but not exported"

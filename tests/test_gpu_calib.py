@@ -85,6 +85,26 @@ def test_precompute_full_size_layer(duo):
     _check(duo, 4096, 2048, 2048, True, seed=11)
 
 
+def test_query_reports_the_context_buffers(duo):
+    """duo_calib_query: the sizes, and buffer addresses whose contents equal
+    what duo_calib_export copies out (read here through duo_copy)."""
+    k, m = 96, 160
+    X = _inputs(k, m, 5)
+    c = duo.Calib(k, m)
+    c.precompute(torch.from_numpy(np.ascontiguousarray(X.T)).cuda(), k // 2)
+    info = c.query()
+    assert info["k"] == k and info["m"] == m
+    lib = duo.load_library()
+    stream = torch.cuda.current_stream().cuda_stream
+    for name, addr, dt, shape in (("perm", "perm_dev", torch.int32, (k,)), ("L", "L_dev", torch.float32, (k, k)),
+                                  ("D", "D_dev", torch.float32, (k, k)), ("col", "col_dev", torch.float32, (k,))):
+        assert info[addr], addr
+        raw = torch.empty(shape, dtype=dt, device="cuda")
+        assert lib.duo_copy(raw.data_ptr(), info[addr], raw.numel() * 4, stream) == 0
+        assert torch.equal(raw, c.get(name)), name
+    c.free()
+
+
 def test_context_reuse_and_errors(duo):
     k, m = 64, 96
     c = duo.Calib(k, m)
