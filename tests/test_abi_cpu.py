@@ -187,3 +187,29 @@ def test_copy_argument_validation(lib):
     assert lib.duo_copy(None, None, 0, None) == 0
     assert lib.duo_copy(FAKE, FAKE, 16, None) in (EINVAL, ECUDA)
 
+
+@pytest.mark.parametrize("cname,pyname,header", [("duo_packed_info", "_Info", "duo.h"),
+                                                  ("duo_calib_info", "_CalibInfo", "duo_calib.h")])
+def test_struct_mirrors_match_the_c_layout(tmp_path, cname, pyname, header):
+    """The ctypes mirrors have the C compiler's size and field offsets
+    (a small C program prints them; gcc, no GPU)."""
+    import shutil
+    import subprocess
+    from paper_2506_20194_gb300 import duo
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    mirror = getattr(duo, pyname)
+    cfields = {"inp": "in"}   # Python keyword renamed in the mirror
+    lines = [f'printf("%zu\\n", sizeof({cname}));']
+    for name, _ in mirror._fields_:
+        lines.append(f'printf("%zu\\n", offsetof({cname}, {cfields.get(name, name)}));')
+    src = tmp_path / "layout.c"
+    src.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "%s"\nint main(void) {\n%s\nreturn 0;\n}\n'
+                   % (header, "\n".join(lines)))
+    exe = tmp_path / "layout"
+    subprocess.run([cc, "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
+    got = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    want = [ctypes.sizeof(mirror)] + [getattr(mirror, name).offset for name, _ in mirror._fields_]
+    assert got == want
+
