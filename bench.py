@@ -158,35 +158,49 @@ def k_of(I, px):
     return (I * (100 - px)) // 100
 
 
-def side_bytes_layer(duo, shape, layer, px):
-    """Companions of the required bytes of one layer step: the kept
-    non-zero values alone (2 sum nnz_j over kept j: the weights loaded, the
-    quantity the paper counts), and the worst case of the required-bytes
-    formula, with the k densest channels of each stage selected instead of
-    the ones x picks; then the values of both as fractions of the dense
-    weights (Fig. 3's loaded fraction and its worst case, App. B.3)."""
+def side_bytes_from_sets(shape, nnz, kept, px):
+    """Companions of the required bytes of one layer step, from the kept
+    channel sets: the kept non-zero values alone (2 sum nnz_j over kept j:
+    the weights loaded, the quantity the paper counts), and the worst case of
+    the required-bytes formula, with the k densest channels of each stage
+    selected instead of the ones x picks; then the values of both as
+    fractions of the dense weights (Fig. 3's loaded fraction and its worst
+    case, App. B.3).  nnz[p]: int64 tensor of non-zeros per input channel of
+    projection p; kept[si]: int64 tensor of stage si's kept channel ids."""
     vals = worst = wvals = dense = 0.0
-    for st, src in zip(STAGES, STAGE_SRC):
+    for si, st in enumerate(STAGES):
         I = shape.I(st[0])
         k = k_of(I, px)
+        for p in st:
+            dense += 2.0 * shape.O(p) * shape.I(p)
         if k == 0:
             worst += 2.0 * I
             continue
-        idx, _ = duo.duo_sparsify(layer["x"][src], k)
-        K = idx.to(torch.int64) & 0xFFFF
-        tot = sum(layer["nnz"][p] for p in st)            # per channel, over the stage's products
+        K = kept[si]
+        tot = sum(nnz[p] for p in st)                    # per channel, over the stage's products
         dense_k = torch.topk(tot, k).indices
         for p in st:
             O = shape.O(p)
-            vals += float(layer["nnz"][p][K].sum().item()) * 2.0
-            wv = float(layer["nnz"][p][dense_k].sum().item()) * 2.0
+            vals += float(nnz[p][K].sum().item()) * 2.0
+            wv = float(nnz[p][dense_k].sum().item()) * 2.0
             wvals += wv
             worst += wv + k * O / 8.0 + 4.0 * O
         worst += 2.0 * I + 4.0 * k
-    for st in STAGES:
-        for p in st:
-            dense += 2.0 * shape.O(p) * shape.I(p)
     return vals, worst, vals / dense, wvals / dense
+
+
+def side_bytes_layer(duo, shape, layer, px):
+    """side_bytes_from_sets with the kept sets from the library's own
+    (parity-tested) sparsifier."""
+    kept = []
+    for st, src in zip(STAGES, STAGE_SRC):
+        k = k_of(shape.I(st[0]), px)
+        if k == 0:
+            kept.append(None)
+            continue
+        idx, _ = duo.duo_sparsify(layer["x"][src], k)
+        kept.append(idx.to(torch.int64) & 0xFFFF)
+    return side_bytes_from_sets(shape, layer["nnz"], kept, px)
 
 
 def required_bytes_layer(duo, shape, layer, px):
