@@ -2,9 +2,10 @@
 plausible error into the oracle for its own duration and checks that the
 pins guarding that part fail. The errors covered: a reversed tie rule,
 ranking by signed value instead of magnitude, a dropped term, a wrong sign,
-a transposed operand, an ignored kept set, mask bits in the wrong order, a
-zero point off by one, a scale rounded through fp32, a sign flip or a
-dropped term in the efficient score, a transposed factor, and the sweep
+a transposed operand, an ignored kept set, a non-strict threshold, mask
+bits in the wrong order, a zero point off by one, a scale rounded through
+fp32, codes rounded half up, a sign flip or a dropped term in the efficient
+score, a transposed factor, no dampening, act_order ignored, and the sweep
 without its activation-sparsity term. Nothing here touches a GPU."""
 import numpy as np
 import pytest
@@ -48,6 +49,16 @@ def test_signed_order_is_caught(monkeypatch):
 
     monkeypatch.setattr(orc, "oracle_sparsify", mutant)
     _fails(pins.test_sparsify_matches_bruteforce, 8)
+
+
+def test_non_strict_threshold_is_caught(monkeypatch):
+    def mutant(x16, tau):   # keeps |x_j| >= |tau| instead of > |tau|
+        x = np.asarray(x16, dtype=np.float16).reshape(-1)
+        K = np.nonzero(np.abs(x.astype(np.float64)) >= abs(float(np.float16(tau))))[0]
+        return K.astype(np.uint16), x[K].copy()
+
+    monkeypatch.setattr(orc, "oracle_sparsify_threshold", mutant)
+    _fails(pins.test_golden_threshold_cases)
 
 
 # ---------------------------------------------------------------- spMspV ----
@@ -125,8 +136,12 @@ def test_zero_point_off_by_one_is_caught(monkeypatch):
     _fails(quant_pins.test_golden_rows)
 
 
-def test_scale_rounded_through_fp32_is_caught(monkeypatch):
-    def mutant(W16, bits):   # the scale's quotient rounded to fp32, then to fp16
+def _rtn_mutant(scale_fp32=False, half_up=False):
+    """The RTN grid with one planted change: the scale's quotient rounded to
+    fp32 before fp16, or codes rounded half up instead of half to even."""
+    rnd = (lambda v: np.floor(v + 0.5)) if half_up else np.rint
+
+    def mutant(W16, bits):
         W = np.asarray(W16, np.float16)
         maxq = (1 << bits) - 1
         O, I = W.shape
@@ -141,20 +156,31 @@ def test_scale_rounded_through_fp32_is_caught(monkeypatch):
             blk = Wd[:, c0:c1]
             lo = np.minimum(blk.min(axis=1), 0.0)
             hi = np.maximum(blk.max(axis=1), 0.0)
-            sg = ((hi - lo) / maxq).astype(np.float32).astype(np.float16)
+            quot = (hi - lo) / maxq
+            sg = (quot.astype(np.float32) if scale_fp32 else quot).astype(np.float16)
             empty = hi == lo
             sg[empty] = np.float16(1.0)
             sg[(sg == 0) & ~empty] = np.uint16(1).view(np.float16)
             sd = sg.astype(np.float64)
-            zg = np.clip(np.rint(-lo / sd), 0, maxq).astype(np.int64)
-            qg = np.clip(np.rint(blk / sd[:, None]) + zg[:, None], 0, maxq).astype(np.int64)
+            zg = np.clip(rnd(-lo / sd), 0, maxq).astype(np.int64)
+            qg = np.clip(rnd(blk / sd[:, None]) + zg[:, None], 0, maxq).astype(np.int64)
             q[:, c0:c1] = np.where(nz[:, c0:c1], qg, 0)
             s16[:, g] = sg
             z[:, g] = zg
         return q, s16, z
 
-    monkeypatch.setattr(orc, "oracle_quantize_rtn", mutant)
+    return mutant
+
+
+def test_scale_rounded_through_fp32_is_caught(monkeypatch):
+    monkeypatch.setattr(orc, "oracle_quantize_rtn", _rtn_mutant(scale_fp32=True))
     _fails(quant_pins.test_golden_rows)
+
+
+def test_codes_rounded_half_up_are_caught(monkeypatch):
+    monkeypatch.setattr(orc, "oracle_quantize_rtn", _rtn_mutant(half_up=True))
+    _fails(quant_pins.test_golden_rows)
+    _fails(quant_pins.test_brute_force_groups, 4)
 
 
 # ----------------------------------------------------------- calibration ----
@@ -182,6 +208,20 @@ def test_dropped_b_is_caught(monkeypatch):
 
 def test_transposed_factor_is_caught(monkeypatch):
     _patch_precompute(monkeypatch, lambda pre: pre.__setitem__("L", pre["L"].T.copy()))
+    _fails(calib_pins.test_invariants_of_L_perm_and_sparse_input)
+
+
+def test_missing_dampening_is_caught(monkeypatch):
+    orig = cal_o.oracle_calib_precompute
+    monkeypatch.setattr(orc, "oracle_calib_precompute",
+                        lambda X, keep, damp=0.1, act_order=True: orig(X, keep, 0.0, act_order))
+    _fails(calib_pins.test_invariants_of_L_perm_and_sparse_input)
+
+
+def test_ignored_act_order_is_caught(monkeypatch):
+    orig = cal_o.oracle_calib_precompute
+    monkeypatch.setattr(orc, "oracle_calib_precompute",
+                        lambda X, keep, damp=0.1, act_order=True: orig(X, keep, damp, False))
     _fails(calib_pins.test_invariants_of_L_perm_and_sparse_input)
 
 
