@@ -48,3 +48,23 @@ def test_two_gloo_ranks_take_the_slowest_time():
     for rank, t, gbs in res:
         assert t == 2.0                                  # max over ranks
         assert gbs == pytest.approx(1e9 * 10 * 2 / 2.0 / 1e9)
+
+
+def test_reference_arm_under_two_ranks_prints_one_line():
+    """bench.py --impl reference launched as the driver launches it for
+    N > 1 (torch.distributed.run, two ranks, gloo on CPU): rank 0 alone runs
+    the oracle and prints one JSON line; the other rank exits 0 silently."""
+    import json
+    import subprocess
+    port = _free_port()
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(port), "bench.py", "--impl", "reference",
+           "--gpus", "2", "--steps", "1", "--warmup", "0"]
+    r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1, r.stdout[-2000:]
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["e2e"]["h2d_bytes_per_step"] == 0
+
