@@ -87,3 +87,90 @@ def test_side_bytes_edge_sparsities():
     vals, worst, frac, wfrac = bench.side_bytes_from_sets(SHAPE, nnz, _kept(x, 100), 100)
     assert vals == 0.0 and frac == 0.0 and wfrac == 0.0
     assert worst == sum(2.0 * SHAPE.I(st[0]) for st in bench.STAGES)
+
+
+BRUTE_SHAPE = synth.llama_shapes(8, 4, 10, "brute")
+
+
+def _brute_layer(seed):
+    """A tiny layer whose products have different per-channel densities, so
+    a shared-input stage's densest set differs from any one product's."""
+    rng = np.random.default_rng(seed)
+    nnz = {}
+    for p in synth.PROJS:
+        O, I = BRUTE_SHAPE.O(p), BRUTE_SHAPE.I(p)
+        keep = rng.random((O, I)) < rng.uniform(0.1, 0.9, size=I)
+        nnz[p] = torch.from_numpy(keep.sum(0).astype(np.int64))
+    return nnz
+
+
+def _check_worst_case_bruteforce(side_bytes, seed, px):
+    """The worst case of the required bytes (App. B.3: the densest channels
+    kept) is the largest required-bytes total over every k-subset of each
+    stage's channels; its value bytes over the dense weights are the
+    worst-case loaded fraction.  Stages are independent, so the per-stage
+    maxima add up."""
+    import itertools
+    nnz = _brute_layer(seed)
+    worst = wvals = dense = 0.0
+    kept = []
+    for st in bench.STAGES:
+        I = BRUTE_SHAPE.I(st[0])
+        k = bench.k_of(I, px)
+        kept.append(torch.arange(k, dtype=torch.int64) if k > 0 else None)
+        best_req = best_vals = None
+        for K in itertools.combinations(range(I), k):
+            v = sum(2.0 * int(nnz[p][j]) for p in st for j in K)
+            req = v + sum(k * BRUTE_SHAPE.O(p) / 8.0 + 4.0 * BRUTE_SHAPE.O(p) for p in st)
+            req += 2.0 * I + 4.0 * k
+            best_req = req if best_req is None else max(best_req, req)
+            best_vals = v if best_vals is None else max(best_vals, v)
+        worst += best_req
+        wvals += best_vals
+        dense += sum(2.0 * BRUTE_SHAPE.O(p) * BRUTE_SHAPE.I(p) for p in st)
+    _, got_worst, _, got_wfrac = side_bytes(BRUTE_SHAPE, nnz, kept, px)
+    assert got_worst == worst, (seed, px)
+    assert got_wfrac == pytest.approx(wvals / dense, rel=1e-12, abs=0.0), (seed, px)
+
+
+@pytest.mark.parametrize("seed", range(4))
+@pytest.mark.parametrize("px", [0, 25, 50, 70])
+def test_worst_case_bytes_bruteforce(seed, px):
+    _check_worst_case_bruteforce(bench.side_bytes_from_sets, seed, px)
+
+
+def test_worst_case_of_one_product_is_caught():
+    """Planted mistake: a shared-input stage takes the densest channels of
+    its first product instead of those of the stage's summed non-zeros."""
+    def mutant(shape, nnz, kept, px):
+        orig_topk = torch.topk
+
+        def topk_first(t, k):   # the stage total swapped for its first product's counts
+            for st in bench.STAGES:
+                if torch.equal(t, sum(nnz[p] for p in st)):
+                    return orig_topk(nnz[st[0]], k)
+            return orig_topk(t, k)
+
+        torch.topk = topk_first
+        try:
+            return bench.side_bytes_from_sets(shape, nnz, kept, px)
+        finally:
+            torch.topk = orig_topk
+
+    with pytest.raises(AssertionError):
+        for seed in range(4):
+            _check_worst_case_bruteforce(mutant, seed, 50)
+
+
+def test_worst_case_without_the_k_cut_is_caught():
+    """Planted mistake: every channel's values counted in the worst case."""
+    def mutant(shape, nnz, kept, px):
+        orig_topk = torch.topk
+        torch.topk = lambda t, k: orig_topk(t, t.numel())
+        try:
+            return bench.side_bytes_from_sets(shape, nnz, kept, px)
+        finally:
+            torch.topk = orig_topk
+
+    with pytest.raises(AssertionError):
+        _check_worst_case_bruteforce(mutant, 0, 50)

@@ -235,3 +235,23 @@ def test_sweep_without_the_activation_term_is_caught(monkeypatch):
 
     monkeypatch.setattr(orc, "oracle_calib_prune_blocked", mutant)
     _fails(calib_pins.test_sweep_blocked_equals_unblocked, 8, 24, 40, 12, 8, 50)
+
+
+# ------------------------------------------------------- byte accounting ----
+
+def test_worst_case_without_the_k_cut_is_caught(monkeypatch):
+    def mutant(nnz_per_channel, k, O, I):   # forgets to keep only k channels
+        n = np.sort(np.asarray(nnz_per_channel, dtype=np.float64))[::-1]
+        return float(n.sum() / (O * I))
+
+    monkeypatch.setattr(orc, "worst_case_loaded_fraction", mutant)
+    _fails(pins.test_worst_case_loaded_fraction_is_the_max_over_kept_sets)
+
+
+def test_worst_case_sparsest_channels_is_caught(monkeypatch):
+    def mutant(nnz_per_channel, k, O, I):   # ascending sort: the k sparsest
+        n = np.sort(np.asarray(nnz_per_channel, dtype=np.float64))
+        return float(n[:k].sum() / (O * I))
+
+    monkeypatch.setattr(orc, "worst_case_loaded_fraction", mutant)
+    _fails(pins.test_worst_case_loaded_fraction_is_the_max_over_kept_sets)

@@ -393,3 +393,26 @@ def test_loaded_fraction_matches_dual_sparsity_product():
         assert abs(f - expect) < 0.01
         assert orc.worst_case_loaded_fraction(nnz, k, O, I) >= f - 1e-12
     assert orc.loaded_fraction(nnz, np.arange(I), O, I) == nnz.sum() / (O * I)
+
+
+def _worst_case_cases():
+    """Tiny layers with channel non-zero counts spread out (distinct enough
+    that the densest, sparsest and first-k sets all differ)."""
+    out = []
+    for seed in range(6):
+        rng = np.random.default_rng(100 + seed)
+        O, I = 7, int(rng.integers(5, 11))
+        keep = rng.random((O, I)) < rng.uniform(0.2, 0.8, size=I)
+        out.append((O, I, keep.sum(0)))
+    return out
+
+
+def test_worst_case_loaded_fraction_is_the_max_over_kept_sets():
+    """App. B.3 bounds the loaded fraction by the case where the k densest
+    channels are the kept ones: over every k-subset K of a tiny layer, the
+    largest Σ_{j∈K} nnz_j / (O I) must equal the function, exactly (integer
+    sums over the same denominator)."""
+    for O, I, nnz in _worst_case_cases():
+        for k in range(I + 1):
+            best = max(sum(int(nnz[j]) for j in K) for K in itertools.combinations(range(I), k))
+            assert orc.worst_case_loaded_fraction(nnz, k, O, I) == best / (O * I), (O, I, k)
