@@ -2,7 +2,7 @@
 // device memory themselves (declared in include/duo.h).
 //
 // duo_pack needs per-record scratch (the non-zero count of every
-// (channel, segment) record, and two totals) and allocates it, plus the
+// (channel, segment) record, and three totals) and allocates it, plus the
 // packed buffers, with cudaMalloc.  Some callers cannot do that: code that
 // runs where the CUDA allocator is off limits (an engine whose device memory
 // all comes from a pool it manages itself, or a process whose allocations
@@ -20,14 +20,17 @@
 
 namespace {
 
-// Scratch limit: I * ceil(O / 1024) records (4 bytes each) plus two 64-bit
-// totals.  262144 records covers, for example, I = 65535 with O <= 4096, or
-// a 28672 x 8192 weight (229376 records).
+// Scratch limit: I * ceil(O / 1024) records (4 bytes each) plus three 64-bit
+// totals that the offset scan writes (16-byte units, non-zeros, the largest
+// record's count).  262144 records covers, for example, I = 65535 with
+// O <= 4096, or a 28672 x 8192 weight (229376 records).
 constexpr int64_t kMaxRecords = DUO_NOALLOC_MAX_RECORDS;
 constexpr size_t kTotalsAt = (size_t)kMaxRecords * 4;
+constexpr size_t kTotalsPad = 256;
+static_assert(kTotalsPad >= 3 * sizeof(unsigned long long), "the scan writes three totals");
 
 // Every GPU that loads the library holds this array until the process exits.
-static __device__ __align__(256) unsigned char g_noalloc_scratch[kTotalsAt + 256];
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kTotalsAt + kTotalsPad];
 
 std::mutex g_mu;
 void* g_scratch_dev[64];
@@ -58,6 +61,16 @@ int scratch_address(void** out) {
 
 bool aligned_to(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// True when the GPU can address p as device memory (device or managed).
+bool on_device(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
 int map_cuda(cudaError_t e) {
   if (e == cudaSuccess) return DUO_OK;
   cudaGetLastError();
@@ -77,17 +90,15 @@ extern "C" int duo_pack_cmb_noalloc(const void* W_fp16_dev, int64_t out, int64_t
   const int64_t S = (out + duo::kSegRows - 1) / duo::kSegRows;
   const int64_t nrec = in * S;
   if (nrec > kMaxRecords) return DUO_ERANGE;
+  if (S > 65535) return DUO_ERANGE;   // segments are a grid dimension, as in duo_pack
   int n = 0;
   if (cudaGetDeviceCount(&n) != cudaSuccess || n <= 0) {
     cudaGetLastError();
     return DUO_ECUDA;
   }
-  cudaPointerAttributes at;
-  if (cudaPointerGetAttributes(&at, W_fp16_dev) != cudaSuccess ||
-      (at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged)) {
-    cudaGetLastError();
+  if (!on_device(W_fp16_dev) || !on_device(off_dev) ||
+      (data_dev != nullptr && !on_device(data_dev)))
     return DUO_EINVAL;
-  }
   void* scratch = nullptr;
   int rc = scratch_address(&scratch);
   if (rc != DUO_OK) return rc;
@@ -98,7 +109,7 @@ extern "C" int duo_pack_cmb_noalloc(const void* W_fp16_dev, int64_t out, int64_t
       reinterpret_cast<unsigned long long*>(static_cast<unsigned char*>(scratch) + kTotalsAt);
 
   // Every scratch word read below is written earlier in the same call (the
-  // count kernel writes all nrec counts, the scan writes both totals), so
+  // count kernel writes all nrec counts, the scan writes all three totals), so
   // nothing needs clearing; the previous call's contents are never read.
   rc = map_cuda(duo::launch_pack_count(W, out, in, ldw, (int)S, cnt, st));
   if (rc != DUO_OK) return rc;
