@@ -23,7 +23,10 @@
  *     stream).  Calls documented "async" only enqueue work on it.
  *   - Channel ids are uint16, so I <= 65535.
  *   - Device-side waits are bounded; a wait that runs out sets a device
- *     status word that duo_device_status() returns (DUO_ETIMEOUT).
+ *     status word (DUO_ETIMEOUT).  Every packed handle has its own word,
+ *     written by the launches whose first handle it is and read by
+ *     duo_packed_status(); duo_device_status() reads every word of the
+ *     device at once.
  *   - There is no host fallback: without a usable CUDA device every compute
  *     entry point returns DUO_ECUDA.
  */
@@ -137,7 +140,7 @@ int duo_sparsify(const void* x_fp16_dev, int64_t in, int64_t k,
  *             x_fp16_dev is ignored and may be NULL.  For BITMASK_Q8 / _Q4
  *             handles the ids must not decrease in id / 128 (ascending ids
  *             do); a list out of that order is rejected on the device
- *             (duo_device_status then returns DUO_EFORMAT).
+ *             (duo_packed_status(h) then returns DUO_EFORMAT).
  *   coded   : BITMASK_Q8 / _Q4 handles need every (handle, 1024-row
  *             segment) pair of the call to have an SM of its own (at most
  *             one per SM of the device, e.g. 152 on a GB300): DUO_ERANGE
@@ -253,7 +256,10 @@ int duo_packed_export(const duo_packed* h, int which, void* dst_host, int64_t by
  *
  * Limits and behaviour:
  *   - in * ceil(out/1024) must not exceed DUO_NOALLOC_MAX_RECORDS (the
- *     scratch holds one 32-bit count per record), else DUO_ERANGE;
+ *     scratch holds one 32-bit count per record), else DUO_ERANGE; so must
+ *     in > 65535 or ceil(out/1024) > 65535, as in duo_pack;
+ *   - W_fp16_dev, off_dev and (when given) data_dev must be device or
+ *     managed memory, else DUO_EINVAL (checked before any device work);
  *   - data_capacity smaller than the packed size: DUO_ERANGE, with
  *     *data_bytes set to the size needed;
  *   - calls no cudaMalloc, cudaFree or other allocating routine;
@@ -288,12 +294,20 @@ int duo_pack_cmb_noalloc(const void* W_fp16_dev, int64_t out, int64_t in, int64_
  */
 int duo_copy(void* dst, const void* src, int64_t bytes, void* stream);
 
-/* Synchronises `stream`, returns and clears the device status word:
- * DUO_OK; DUO_ETIMEOUT if a bounded device wait ran out since the last
- * call; DUO_EFORMAT if a kernel met a record size or channel id outside the
- * format's bounds (the affected work was skipped); DUO_ECUDA if the stream
- * reports an error. */
+/* Synchronises `stream`, returns and clears the device status words of the
+ * current device (the process-wide word and the word of every live handle
+ * on it): DUO_OK; DUO_ETIMEOUT if a bounded device wait ran out since the
+ * words were last read; DUO_EFORMAT if a kernel met a record size or channel
+ * id outside the format's bounds (the affected work was skipped); DUO_ECUDA
+ * if the stream reports an error. */
 int duo_device_status(void* stream);
+
+/* duo_packed_status -- the same for one handle's word only: the status of
+ * the launches whose first (or only) handle h is, since the word was last
+ * read.  Synchronises `stream`.  Launches on other handles, or on other
+ * streams, do not report here.  Errors: DUO_EINVAL (NULL or freed h),
+ * DUO_ECUDA. */
+int duo_packed_status(const duo_packed* h, void* stream);
 
 /* Text of a status code (static storage). */
 const char* duo_strerror(int code);

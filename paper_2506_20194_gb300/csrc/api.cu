@@ -5,6 +5,7 @@
 #include <mutex>
 #include <new>
 #include <unordered_set>
+#include <vector>
 
 #include <cuda_runtime.h>
 
@@ -31,7 +32,8 @@ struct duo_packed {
   void* data;
   int64_t data_bytes;
   int vbits;           // BITMASK formats: bits per stored value (16, 8, 4)
-  unsigned int* sync;  // BITMASK: 2-word grid barrier of the spMspV kernel
+  unsigned int* sync;  // 256 zeroed bytes: {count, generation} of the spMspV kernel's
+                       // grid barrier, then the handle's device status word
   uint16_t* kept;      // BITMASK: room for a kept list (ids, then values; 2 x in each)
   int max_record;      // BITMASK: bytes of the largest record
 };
@@ -205,8 +207,8 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
       if (e != cudaSuccess) return fail(map_err(e));
     }
     h->index_bytes = (int64_t)sizeof(uint32_t) * (in * S + 1);
-    // The offsets are followed (at a 256-byte boundary) by the two barrier
-    // words of the spMspV kernel, zeroed here.
+    // The offsets are followed (at a 256-byte boundary) by the grid-barrier
+    // words of the spMspV kernel and the handle's status word, zeroed here.
     const size_t sync_at = (size_t)(h->index_bytes + 255) / 256 * 256;
     // after the offsets: the grid barrier words, then a kept-list buffer for
     // launches with more (product, segment) runs than SMs (selection first)
@@ -235,7 +237,12 @@ int duo_pack(const void* W_fp16_dev, int64_t out, int64_t in, int64_t ldw, int f
     h->nseg = 0;
     h->index_bytes = (int64_t)sizeof(uint64_t) * (in + 1);
     h->aux_bytes = (int64_t)sizeof(uint32_t) * in;
-    e = duo_malloc(&index, (size_t)h->index_bytes);
+    // the column pointers, then (at a 256-byte boundary) the status block
+    const size_t sync_at = (size_t)(h->index_bytes + 255) / 256 * 256;
+    e = duo_malloc(&index, sync_at + 256);
+    if (e != cudaSuccess) return fail(map_err(e));
+    h->sync = reinterpret_cast<unsigned int*>(static_cast<char*>(index) + sync_at);
+    e = cudaMemsetAsync(h->sync, 0, 256, st);
     if (e != cudaSuccess) return fail(map_err(e));
     e = duo_malloc(&aux, (size_t)h->aux_bytes);
     if (e != cudaSuccess) return fail(map_err(e));
@@ -329,6 +336,7 @@ int duo_spmspv_threshold(const duo_packed* const* hs, int n, const void* x_fp16_
   a.tau_key = tau_fp16 & 0x7FFFu;
   a.vbits = hs[0]->vbits;
   a.bar = hs[0]->sync;
+  a.status = hs[0]->sync + 2;
   a.slot_bytes = 0;
   for (int p = 0; p < n; ++p) {
     a.slot_bytes = hs[p]->max_record > a.slot_bytes ? hs[p]->max_record : a.slot_bytes;
@@ -346,8 +354,16 @@ int duo_spmspv_threshold(const duo_packed* const* hs, int n, const void* x_fp16_
   return map_err(e);
 }
 
+// Launch options other than the defaults (the failure-detection test only):
+// a wait limit and the grid-barrier words to use.
+struct LaunchOpts {
+  unsigned long long wait_ns;
+  unsigned int* bar;
+};
+
 static int spmspv_common(const duo_packed* const* hs, int n, const void* x, const uint16_t* kidx,
-                         const void* kval, int64_t k, float* const* ys, void* stream) {
+                         const void* kval, int64_t k, float* const* ys, void* stream,
+                         const LaunchOpts* opt = nullptr) {
   if (hs == nullptr || ys == nullptr || n < 1 || n > duo::kMaxProblems) return DUO_EINVAL;
   const bool listed = kidx != nullptr || kval != nullptr;
   if (k != 0) {   // with k == 0 nothing is read: y = 0 whatever the input pointers
@@ -388,7 +404,9 @@ static int spmspv_common(const duo_packed* const* hs, int n, const void* x, cons
     a.x = static_cast<const uint16_t*>(x);
     a.kidx = listed ? kidx : nullptr;
     a.kval = listed ? static_cast<const uint16_t*>(kval) : nullptr;
-    a.bar = hs[0]->sync;
+    a.bar = opt ? opt->bar : hs[0]->sync;
+    a.status = hs[0]->sync + 2;
+    a.wait_ns = opt ? opt->wait_ns : 0;
     a.slot_bytes = 0;
     for (int p = 0; p < n; ++p) a.slot_bytes = hs[p]->max_record > a.slot_bytes ? hs[p]->max_record : a.slot_bytes;
     for (int p = 0; p < n; ++p) {
@@ -417,6 +435,7 @@ static int spmspv_common(const duo_packed* const* hs, int n, const void* x, cons
   } else {
     const duo_packed* h = hs[0];
     duo::Idx16Args a{};
+    a.status = h->sync + 2;
     a.data = static_cast<const uint8_t*>(h->data);
     a.colptr = static_cast<const uint64_t*>(h->index);
     a.cnt = static_cast<const uint32_t*>(h->aux);
@@ -502,6 +521,28 @@ int duo_packed_export(const duo_packed* h, int which, void* dst_host, int64_t by
   return map_err(cudaMemcpy(dst_host, src, (size_t)n, cudaMemcpyDeviceToHost));
 }
 
+namespace {
+
+// Reads and clears one handle's device status word (stream synchronised).
+int take_handle_status(const duo_packed* h, unsigned int* out) {
+  unsigned int v = 0, zero = 0;
+  if (cudaMemcpy(&v, h->sync + 2, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess ||
+      cudaMemcpy(h->sync + 2, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) {
+    cudaGetLastError();
+    return DUO_ECUDA;
+  }
+  *out = v;
+  return DUO_OK;
+}
+
+int status_code(unsigned int st) {
+  if (st & 1u) return DUO_ETIMEOUT;
+  if (st & 2u) return DUO_EFORMAT;
+  return DUO_OK;
+}
+
+}  // namespace
+
 int duo_device_status(void* stream) {
   int rc = cuda_ready();
   if (rc != DUO_OK) return rc;
@@ -510,9 +551,68 @@ int duo_device_status(void* stream) {
   unsigned int st = 0;
   e = duo::read_and_clear_status(&st);
   if (e != cudaSuccess) return DUO_ECUDA;
-  if (st & 1u) return DUO_ETIMEOUT;
-  if (st & 2u) return DUO_EFORMAT;
-  return DUO_OK;
+  std::vector<const duo_packed*> hs;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    hs.assign(live_handles().begin(), live_handles().end());
+  }
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return DUO_ECUDA;
+  for (const duo_packed* h : hs) {
+    if (h->device != dev) continue;
+    unsigned int v = 0;
+    rc = take_handle_status(h, &v);
+    if (rc != DUO_OK) return rc;
+    st |= v;
+  }
+  return status_code(st);
+}
+
+int duo_packed_status(const duo_packed* h, void* stream) {
+  if (h == nullptr || !is_live(h)) return DUO_EINVAL;
+  int rc = cuda_ready();
+  if (rc != DUO_OK) return rc;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) {
+    cudaGetLastError();
+    return DUO_ECUDA;
+  }
+  unsigned int v = 0;
+  rc = take_handle_status(h, &v);
+  if (rc != DUO_OK) return rc;
+  return status_code(v);
+}
+
+// Internal, for the failure-detection test only (not declared in duo.h):
+// the fused product with every bounded wait limited to wait_ns and a grid
+// barrier that cannot open (its own words, the count preset so far above
+// the grid size that no arrival is the last), so every CTA gives up at its
+// first reduction into y and reports DUO_ETIMEOUT through the handle's
+// status word.  y is left undefined; the handle's own barrier words are
+// not touched.
+int duo_test_spmspv_blocked(const duo_packed* h, const void* x_fp16_dev, int64_t k, float* y_dev,
+                            unsigned long long wait_ns, void* stream) {
+  if (h == nullptr || !is_live(h) || !is_cmb(h->fmt)) return DUO_EINVAL;
+  if (wait_ns == 0 || wait_ns > 100000000ull) return DUO_EINVAL;   // at most 0.1 s
+  int rc = cuda_ready();
+  if (rc != DUO_OK) return rc;
+  void* bar = nullptr;
+  cudaError_t e = cudaMalloc(&bar, 256);
+  if (e != cudaSuccess) return map_err(e);
+  const unsigned int preset[2] = {0x80000000u, 0u};
+  e = cudaMemset(bar, 0, 256);
+  if (e == cudaSuccess) e = cudaMemcpy(bar, preset, sizeof(preset), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    cudaFree(bar);
+    return map_err(e);
+  }
+  const duo_packed* hs[1] = {h};
+  float* ys[1] = {y_dev};
+  const LaunchOpts opt = {wait_ns, static_cast<unsigned int*>(bar)};
+  rc = spmspv_common(hs, 1, x_fp16_dev, nullptr, nullptr, k, ys, stream, &opt);
+  cudaError_t e2 = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  cudaFree(bar);
+  if (rc != DUO_OK) return rc;
+  return map_err(e2);
 }
 
 }  // extern "C"

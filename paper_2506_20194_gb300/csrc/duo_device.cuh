@@ -16,10 +16,12 @@ constexpr int MAX_RECORD_BYTES = MASK_BYTES + 2 * SEG_ROWS;  // 2176
 constexpr int MAXP = 4;                  // products per multi launch
 constexpr uint64_t WAIT_LIMIT_NS = 1000000000ull;  // 1 s per bounded wait
 
-// Device status word (bit 0: a bounded wait ran out; bit 1: a record size or
-// channel id outside the format's bounds), read by duo_device_status.  The
-// translation unit that owns it (kernels.cu) defines DUO_STATUS_OWNER; any
-// other unit including this header gets a private copy nobody reads.
+// Device status words (bit 0: a bounded wait ran out; bit 1: a record size
+// or channel id outside the format's bounds).  A launch with a packed handle
+// writes that handle's word (kept next to its grid-barrier words); the
+// process-wide word below is for kernels without a handle.  The translation
+// unit that owns it (kernels.cu) defines DUO_STATUS_OWNER; any other unit
+// including this header gets a private copy nobody reads.
 #ifdef DUO_STATUS_OWNER
 __device__ unsigned int g_status = 0u;
 #else
@@ -85,17 +87,19 @@ __device__ __forceinline__ bool mbar_try_wait_suspend(uint64_t* bar, uint32_t pa
 constexpr uint32_t SUSPEND_HINT_NS = 2000;
 
 // Waits for the phase of `parity` with a wall-clock limit.  On timeout the
-// device status word and the CTA's abort flag are set and false returned;
-// a wait also gives up (false) once another warp has raised the abort flag.
+// status word (bit STATUS_TIMEOUT) and the CTA's abort flag are set and
+// false returned; a wait also gives up (false) once another warp has raised
+// the abort flag.
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity,
-                                                  volatile int* abort_flag) {
+                                                  volatile int* abort_flag, unsigned int* status,
+                                                  uint64_t limit_ns = WAIT_LIMIT_NS) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   while (true) {
     if (mbar_try_wait_suspend(bar, parity, SUSPEND_HINT_NS)) return true;
     if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
-      atomicOr(&g_status, STATUS_TIMEOUT);
+    if (globaltimer_ns() - t0 > limit_ns) {
+      atomicOr(status, STATUS_TIMEOUT);
       *abort_flag = 1;
       return false;
     }
@@ -103,11 +107,12 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
 }
 
 // Same, without an abort flag (used while draining after an abort).
-__device__ __forceinline__ bool mbar_wait_limited(uint64_t* bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait_limited(uint64_t* bar, uint32_t parity, unsigned int* status,
+                                                   uint64_t limit_ns = WAIT_LIMIT_NS) {
   const uint64_t t0 = globaltimer_ns();
   while (!mbar_try_wait(bar, parity)) {
-    if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
-      atomicOr(&g_status, STATUS_TIMEOUT);
+    if (globaltimer_ns() - t0 > limit_ns) {
+      atomicOr(status, STATUS_TIMEOUT);
       return false;
     }
   }
@@ -123,6 +128,11 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       "[%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
       "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
       : "memory");
+}
+
+// L2 prefetch of the 128-byte line holding p (any alignment).
+__device__ __forceinline__ void prefetch_line_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
 }
 
 // L2 prefetch of [src, src + bytes) (16-byte aligned, bytes % 16 == 0).
@@ -166,23 +176,6 @@ __device__ __forceinline__ int ld_acquire_cta_shared(const int* p) {
 
 __device__ __forceinline__ void st_release_cta_shared(int* p, int v) {
   asm volatile("st.release.cta.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
-}
-
-// Spins (bounded, like mbar_wait_bounded) until the shared word at p equals
-// want.  Used to check the exact identity of a ring slot's fill, which an
-// mbarrier parity alone cannot tell apart from a fill two phases earlier.
-__device__ __forceinline__ bool wait_shared_eq(const int* p, int want, volatile int* abort_flag) {
-  if (ld_acquire_cta_shared(p) == want) return true;
-  const uint64_t t0 = globaltimer_ns();
-  while (true) {
-    if (ld_acquire_cta_shared(p) == want) return true;
-    if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
-      atomicOr(&g_status, STATUS_TIMEOUT);
-      *abort_flag = 1;
-      return false;
-    }
-  }
 }
 
 // Programmatic dependent launch: wait until the previous kernel of the
@@ -343,6 +336,7 @@ struct SelShared {
   uint32_t hist[SEL_BINS];
   uint32_t sub[16];               // keys of bin C by key & 15
   uint32_t wcnt[SEL_MAX_WARPS];   // per-warp counts
+  uint32_t tmp[6 * SEL_MAX_WARPS];   // select_window's scratch
   uint32_t C, aboveC;
   int T, cut;                     // the selection's result (see select_threshold)
 };
@@ -359,103 +353,50 @@ __device__ __forceinline__ void select_clear(SelShared* sh) {
 // Inf).
 __device__ __forceinline__ int key_of(const uint16_t* xs, int j) { return xs[j] & 0x7FFF; }
 
-// Exact top-k by magnitude (§3) as a threshold: keeps the k channels with
-// the largest |x_j|, ties to the lower index.  On return (to every thread)
-// channel j is kept iff key_j > T, or key_j == T and j <= cut.
-//
-//  1. histogram of key >> 4 (2048 bins, shared-memory atomics);
-//  2. one warp finds the bin C where the count from the top reaches k: a
-//     suffix scan over 32 lanes x 64 bins, then over the 64 bins of the
-//     crossing lane (2 per lane);
-//  3. histogram of key & 15 over the keys of bin C (few: contention-free
-//     atomics);
-//  4. one warp gets T = 16 C + b and q = k - count(key > T), the number of
-//     channels with key == T to keep (the lowest-indexed ones);
-//  5. only if fewer than all of them are kept: each warp counts the ties in
-//     its contiguous run of 32-channel words, and the warp holding the q-th
-//     tie finds its channel, cut; otherwise cut = I.
-// k <= 0 keeps nothing (T = 0x7FFF, cut = -1), k >= I everything (T = -1).
-// xs holds the fp16 bits of x (room for a whole number of 32-channel words);
-// select_clear() and the loading of xs come first, then a __syncthreads.  All
-// threads of the block take part (512 <= blockDim.x <= 1024, a multiple of
-// 32); it ends with a __syncthreads.
-__device__ inline void select_threshold(const uint16_t* xs, int I, int k, SelShared* sh, int* T_out,
-                                        int* cut_out) {
-  const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, wid = tid >> 5;
-  const int nwarps = nt >> 5;
+// Step 2 of select_threshold, by warp 0 only (after the histogram of key >> 4
+// is complete): the bin C where the count of keys from the top reaches k,
+// and the number of keys above it, into sh->C and sh->aboveC.  1 <= k < I.
+__device__ __forceinline__ void select_find_bin(SelShared* sh, uint32_t kk, int lane) {
+  const uint4* h4 = reinterpret_cast<const uint4*>(sh->hist) + 16 * lane;
+  uint32_t s64 = 0;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const uint4 h = h4[(i + lane) & 15];   // rotated: a quarter warp hits 8 bank groups
+    s64 += (h.x + h.y) + (h.z + h.w);
+  }
+  uint32_t sl = s64;   // keys in bins >= 64 * lane
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t t = __shfl_down_sync(FULL_MASK, sl, o);
+    if (lane + o < 32) sl += t;
+  }
+  const int L = 31 - __clz(__ballot_sync(FULL_MASK, sl >= kk));
+  const uint32_t above_l = __shfl_sync(FULL_MASK, sl - s64, L);   // keys in bins >= 64 (L + 1)
+  const uint2 h2 = reinterpret_cast<const uint2*>(sh->hist)[32 * L + lane];   // bins 64 L + 2 lane, +1
+  const uint32_t s2 = h2.x + h2.y;
+  uint32_t sp = s2;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t t = __shfl_down_sync(FULL_MASK, sp, o);
+    if (lane + o < 32) sp += t;
+  }
+  const int M = 31 - __clz(__ballot_sync(FULL_MASK, above_l + sp >= kk));
+  if (lane == M) {
+    const uint32_t above = above_l + sp - s2;   // keys above bin 64 L + 2 M + 1
+    const bool hi = above + h2.y >= kk;
+    sh->C = 64u * (uint32_t)L + 2u * (uint32_t)M + (hi ? 1u : 0u);
+    sh->aboveC = hi ? above : above + h2.y;
+  }
+}
+
+// Steps 4 and 5 of select_threshold (after the histogram of key & 15 over
+// the keys of bin C is complete): T, and the tie cut when fewer than all
+// keys equal to T are kept.  Every thread of the block calls it; it ends
+// with a __syncthreads.
+__device__ inline void select_finish(const uint16_t* xs, int I, int k, SelShared* sh, int* T_out,
+                                     int* cut_out) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   const uint32_t kk = (uint32_t)k;
-  if (k <= 0 || k >= I) {
-    *T_out = k <= 0 ? 0x7FFF : -1;   // no key exceeds 0x7FFF; every key exceeds -1
-    *cut_out = -1;
-    __syncthreads();
-    return;
-  }
-  // 1. histogram of the high 11 key bits (4 independent loads in flight)
-  {
-    int j = tid;
-    for (; j + 3 * nt < I; j += 4 * nt) {
-      const int k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
-      const int k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
-      atomicAdd(&sh->hist[k0 >> 4], 1u);
-      atomicAdd(&sh->hist[k1 >> 4], 1u);
-      atomicAdd(&sh->hist[k2 >> 4], 1u);
-      atomicAdd(&sh->hist[k3 >> 4], 1u);
-    }
-    for (; j < I; j += nt) atomicAdd(&sh->hist[key_of(xs, j) >> 4], 1u);
-  }
-  __syncthreads();
-  // 2. threshold bin C, by warp 0
-  if (wid == 0) {
-    const uint4* h4 = reinterpret_cast<const uint4*>(sh->hist) + 16 * lane;
-    uint32_t s64 = 0;
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const uint4 h = h4[(i + lane) & 15];   // rotated: a quarter warp hits 8 bank groups
-      s64 += (h.x + h.y) + (h.z + h.w);
-    }
-    uint32_t sl = s64;   // keys in bins >= 64 * lane
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t t = __shfl_down_sync(FULL_MASK, sl, o);
-      if (lane + o < 32) sl += t;
-    }
-    const int L = 31 - __clz(__ballot_sync(FULL_MASK, sl >= kk));
-    const uint32_t above_l = __shfl_sync(FULL_MASK, sl - s64, L);   // keys in bins >= 64 (L + 1)
-    const uint2 h2 = reinterpret_cast<const uint2*>(sh->hist)[32 * L + lane];   // bins 64 L + 2 lane, +1
-    const uint32_t s2 = h2.x + h2.y;
-    uint32_t sp = s2;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t t = __shfl_down_sync(FULL_MASK, sp, o);
-      if (lane + o < 32) sp += t;
-    }
-    const int M = 31 - __clz(__ballot_sync(FULL_MASK, above_l + sp >= kk));
-    if (lane == M) {
-      const uint32_t above = above_l + sp - s2;   // keys above bin 64 L + 2 M + 1
-      const bool hi = above + h2.y >= kk;
-      sh->C = 64u * (uint32_t)L + 2u * (uint32_t)M + (hi ? 1u : 0u);
-      sh->aboveC = hi ? above : above + h2.y;
-    }
-  }
-  __syncthreads();
-  // 3. the 16 keys of bin C
-  {
-    const int C = (int)sh->C;
-    int j = tid;
-    for (; j + 3 * nt < I; j += 4 * nt) {
-      const int k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
-      const int k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
-      if ((k0 >> 4) == C) atomicAdd(&sh->sub[k0 & 15], 1u);
-      if ((k1 >> 4) == C) atomicAdd(&sh->sub[k1 & 15], 1u);
-      if ((k2 >> 4) == C) atomicAdd(&sh->sub[k2 & 15], 1u);
-      if ((k3 >> 4) == C) atomicAdd(&sh->sub[k3 & 15], 1u);
-    }
-    for (; j < I; j += nt) {
-      const int key = key_of(xs, j);
-      if ((key >> 4) == C) atomicAdd(&sh->sub[key & 15], 1u);
-    }
-  }
-  __syncthreads();
   // 4. T and q (lane v < 16 = key & 15 inside bin C), by every warp: the
   //    result is read by all, with no further barrier.
   int T, q, ties;
@@ -509,6 +450,74 @@ __device__ inline void select_threshold(const uint16_t* xs, int I, int k, SelSha
   __syncthreads();
 }
 
+// Exact top-k by magnitude (§3) as a threshold: keeps the k channels with
+// the largest |x_j|, ties to the lower index.  On return (to every thread)
+// channel j is kept iff key_j > T, or key_j == T and j <= cut.
+//
+//  1. histogram of key >> 4 (2048 bins, shared-memory atomics);
+//  2. one warp finds the bin C where the count from the top reaches k: a
+//     suffix scan over 32 lanes x 64 bins, then over the 64 bins of the
+//     crossing lane (2 per lane);
+//  3. histogram of key & 15 over the keys of bin C (few: contention-free
+//     atomics);
+//  4. one warp gets T = 16 C + b and q = k - count(key > T), the number of
+//     channels with key == T to keep (the lowest-indexed ones);
+//  5. only if fewer than all of them are kept: each warp counts the ties in
+//     its contiguous run of 32-channel words, and the warp holding the q-th
+//     tie finds its channel, cut; otherwise cut = I.
+// k <= 0 keeps nothing (T = 0x7FFF, cut = -1), k >= I everything (T = -1).
+// xs holds the fp16 bits of x (room for a whole number of 32-channel words);
+// select_clear() and the loading of xs come first, then a __syncthreads.  All
+// threads of the block take part (512 <= blockDim.x <= 1024, a multiple of
+// 32); it ends with a __syncthreads.
+__device__ inline void select_threshold(const uint16_t* xs, int I, int k, SelShared* sh, int* T_out,
+                                        int* cut_out) {
+  const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, wid = tid >> 5;
+  const uint32_t kk = (uint32_t)k;
+  if (k <= 0 || k >= I) {
+    *T_out = k <= 0 ? 0x7FFF : -1;   // no key exceeds 0x7FFF; every key exceeds -1
+    *cut_out = -1;
+    __syncthreads();
+    return;
+  }
+  // 1. histogram of the high 11 key bits (4 independent loads in flight)
+  {
+    int j = tid;
+    for (; j + 3 * nt < I; j += 4 * nt) {
+      const int k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
+      const int k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
+      atomicAdd(&sh->hist[k0 >> 4], 1u);
+      atomicAdd(&sh->hist[k1 >> 4], 1u);
+      atomicAdd(&sh->hist[k2 >> 4], 1u);
+      atomicAdd(&sh->hist[k3 >> 4], 1u);
+    }
+    for (; j < I; j += nt) atomicAdd(&sh->hist[key_of(xs, j) >> 4], 1u);
+  }
+  __syncthreads();
+  // 2. threshold bin C, by warp 0
+  if (wid == 0) select_find_bin(sh, kk, lane);
+  __syncthreads();
+  // 3. the 16 keys of bin C
+  {
+    const int C = (int)sh->C;
+    int j = tid;
+    for (; j + 3 * nt < I; j += 4 * nt) {
+      const int k0 = key_of(xs, j), k1 = key_of(xs, j + nt);
+      const int k2 = key_of(xs, j + 2 * nt), k3 = key_of(xs, j + 3 * nt);
+      if ((k0 >> 4) == C) atomicAdd(&sh->sub[k0 & 15], 1u);
+      if ((k1 >> 4) == C) atomicAdd(&sh->sub[k1 & 15], 1u);
+      if ((k2 >> 4) == C) atomicAdd(&sh->sub[k2 & 15], 1u);
+      if ((k3 >> 4) == C) atomicAdd(&sh->sub[k3 & 15], 1u);
+    }
+    for (; j < I; j += nt) {
+      const int key = key_of(xs, j);
+      if ((key >> 4) == C) atomicAdd(&sh->sub[key & 15], 1u);
+    }
+  }
+  __syncthreads();
+  select_finish(xs, I, k, sh, T_out, cut_out);
+}
+
 // Writes the channels j in [c0, c1) that a threshold keeps (key_j > T, or
 // key_j == T and j <= cut) in ascending order to klist[0..n) (and their fp16
 // bits to kvals if given) and returns n to every thread.  Warps take
@@ -549,6 +558,223 @@ __device__ inline int thresh_compact(const uint16_t* xs, int c0, int c1, int T, 
   }
   __syncthreads();
   return (int)total;
+}
+
+// Whether select_window<..., NT>() can hold this x in registers: 16-byte
+// aligned, at most four 16-byte chunks per thread.
+template <int NT>
+__device__ __forceinline__ bool select_window_ok(const uint16_t* x, int I) {
+  return (reinterpret_cast<uintptr_t>(x) & 15u) == 0 && (I >> 3) <= 4 * NT;
+}
+
+// x into shared memory (fp16 bits), the kept set, and this CTA's share of
+// the kept list, all from registers: each thread holds NCH 16-byte chunks
+// of x (chunk c of thread t: channels 8 (t + c NT) .. + 7; the last
+// I % 8 channels, one per thread, after them).
+//  * top-k: a histogram of key >> 4 (2048 bins) counted straight from the
+//    registers; every warp finds the bin C where the count from the top
+//    reaches k (each warp sums 128 bins; then each warp reads the crossing
+//    warp's bins again); the keys of bin C give T = 16 C + b, and q, the
+//    number of channels with key == T to keep (the lowest-indexed ones).
+//    The threshold mask keeps key > tau (T = tau, q = 0).
+//  * one block scan of per-chunk counts of key > T and key == T (in channel
+//    order) ranks every channel: a kept channel (key > T, or key == T with
+//    fewer than q equal keys before it) has rank #(key > T before it) +
+//    min(q, #(key == T before it)); each thread writes its kept channels
+//    whose rank lies in this CTA's window [K m / nr, K (m + 1) / nr), K the
+//    number kept, to klist (ascending).  Every CTA of a run thus gets the
+//    same number of channels (+-1) however x is spread.
+// Returns the window size; ends with a barrier.  NCH = ceil((I / 8) /
+// NT), 1..4 (select_window_ok() tells whether it fits).  All NT threads of the
+// block take part; tmp needs 6 NT / 32 words.
+template <bool TOPK, int NCH, int NT>
+__device__ __noinline__ int select_window(const uint16_t* x, int I, int k, int tau_key,
+                                             uint16_t* xs, SelShared* sh, uint32_t m, uint32_t nr,
+                                             uint16_t* klist, uint32_t* tmp) {
+  constexpr int ST_THREADS = NT, ST_WARPS = NT / 32;
+  static_assert(ST_WARPS * 128 == SEL_BINS, "each warp sums 128 histogram bins");
+  static_assert(NCH * 8 <= 32 && NCH >= 1, "at most four chunks (32 channels) a thread");
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int nvec = I >> 3;
+  const uint4* x4 = reinterpret_cast<const uint4*>(x);
+  uint32_t w[4 * NCH];   // the chunks, 2 channels per word
+  bool have[NCH];
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) {
+    const int i = tid + c * ST_THREADS;
+    have[c] = i < nvec;
+    const uint4 v = have[c] ? __ldg(x4 + i) : make_uint4(0u, 0u, 0u, 0u);
+    w[4 * c] = v.x;
+    w[4 * c + 1] = v.y;
+    w[4 * c + 2] = v.z;
+    w[4 * c + 3] = v.w;
+    if (have[c]) reinterpret_cast<uint4*>(xs)[i] = v;
+  }
+  const int jt = (nvec << 3) + tid;   // the tail channel of this thread, if < I
+  const bool tail = jt < I;
+  const uint16_t xt = tail ? x[jt] : (uint16_t)0;
+  if (tail) xs[jt] = xt;
+  auto key_at = [&](int c, int h) { return (int)((w[4 * c + (h >> 1)] >> (16 * (h & 1))) & 0x7FFFu); };
+  int T, q = 0;
+  if (!TOPK) {
+    T = tau_key;
+  } else if (k <= 0 || k >= I) {
+    T = k <= 0 ? 0x7FFF : -1;
+  } else {
+    const uint32_t kk = (uint32_t)k;
+#pragma unroll
+    for (int c = 0; c < NCH; ++c)
+      if (have[c])
+#pragma unroll
+        for (int h = 0; h < 8; ++h) atomicAdd(&sh->hist[key_at(c, h) >> 4], 1u);
+    if (tail) atomicAdd(&sh->hist[(xt & 0x7FFFu) >> 4], 1u);
+    __syncthreads();
+    // bin C: warp v sums bins 128 v .. 128 v + 127; every warp then scans the
+    // 16 sums and the crossing warp's bins (lane l: bins 4 l .. 4 l + 3)
+    {
+      const uint4 h4 = reinterpret_cast<const uint4*>(sh->hist)[32 * wid + lane];
+      const uint32_t wsum = __reduce_add_sync(FULL_MASK, (h4.x + h4.y) + (h4.z + h4.w));
+      if (lane == 0) tmp[wid] = wsum;
+    }
+    __syncthreads();
+    {
+      const uint32_t wv = lane < ST_WARPS ? tmp[lane] : 0u;
+      uint32_t suf = wv;   // keys in bins >= 128 lane
+#pragma unroll
+      for (int o = 1; o < ST_WARPS; o <<= 1) {
+        const uint32_t t = __shfl_down_sync(FULL_MASK, suf, o);
+        if (lane + o < ST_WARPS) suf += t;
+      }
+      const int W = 31 - __clz(__ballot_sync(FULL_MASK, lane < ST_WARPS && suf >= kk));
+      const uint32_t above_w = __shfl_sync(FULL_MASK, suf - wv, W);   // keys above warp W's bins
+      const uint4 h4 = reinterpret_cast<const uint4*>(sh->hist)[32 * W + lane];
+      const uint32_t s4 = (h4.x + h4.y) + (h4.z + h4.w);
+      uint32_t ls = s4;   // keys in warp W's bins >= 4 lane
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t t = __shfl_down_sync(FULL_MASK, ls, o);
+        if (lane + o < 32) ls += t;
+      }
+      const int L = 31 - __clz(__ballot_sync(FULL_MASK, above_w + ls >= kk));
+      uint32_t above = above_w + ls - s4;   // keys above bin 4 L + 3 of warp W
+      int b = 3;
+      if (above + h4.w < kk) {
+        above += h4.w;
+        b = 2;
+        if (above + h4.z < kk) {
+          above += h4.z;
+          b = 1;
+          if (above + h4.y < kk) {
+            above += h4.y;
+            b = 0;
+          }
+        }
+      }
+      const int C = 128 * W + 4 * L + __shfl_sync(FULL_MASK, b, L);
+      const uint32_t aboveC = __shfl_sync(FULL_MASK, above, L);
+      // the keys of bin C, by their low 4 bits
+#pragma unroll
+      for (int c = 0; c < NCH; ++c)
+        if (have[c])
+#pragma unroll
+          for (int h = 0; h < 8; ++h) {
+            const int key = key_at(c, h);
+            if ((key >> 4) == C) atomicAdd(&sh->sub[key & 15], 1u);
+          }
+      if (tail && (int)((xt & 0x7FFFu) >> 4) == C) atomicAdd(&sh->sub[xt & 15u], 1u);
+      __syncthreads();
+      // T and q, in every warp: the 16 keys of bin C from the top
+      const uint32_t sv = lane < 16 ? sh->sub[lane] : 0u;
+      uint32_t sfx = sv;   // keys of bin C with key & 15 >= lane
+#pragma unroll
+      for (int o = 1; o < 16; o <<= 1) {
+        const uint32_t t = __shfl_down_sync(FULL_MASK, sfx, o);
+        if (lane + o < 16) sfx += t;
+      }
+      const uint32_t need = kk - aboveC;   // >= 1
+      const int bb = 31 - __clz(__ballot_sync(FULL_MASK, lane < 16 && sfx >= need));
+      T = 16 * C + bb;
+      q = (int)(need - __shfl_sync(FULL_MASK, sfx - sv, bb));   // >= 1
+    }
+  }
+  // per chunk: bits and counts of key > T and key == T
+  uint32_t gb[NCH], eb[NCH];
+  uint32_t p[5] = {0u, 0u, 0u, 0u, 0u};   // gt of chunks 0|1, 2|3, eq 0|1, 2|3, {gt, eq} of the tail
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) {
+    uint32_t g = 0, e = 0;
+    if (have[c])
+#pragma unroll
+      for (int h = 0; h < 8; ++h) {
+        const int key = key_at(c, h);
+        g |= (key > T ? 1u : 0u) << h;
+        e |= (key == T ? 1u : 0u) << h;
+      }
+    gb[c] = g;
+    eb[c] = e;
+    p[c >> 1] |= (uint32_t)__popc(g) << (16 * (c & 1));
+    p[2 + (c >> 1)] |= (uint32_t)__popc(e) << (16 * (c & 1));
+  }
+  const int tkey = (int)(xt & 0x7FFFu);
+  const uint32_t tg = (tail && tkey > T) ? 1u : 0u, te = (tail && tkey == T) ? 1u : 0u;
+  p[4] = tg | (te << 16);
+  // block exclusive scan of the five packed counters (16-bit fields: at
+  // most 8 ST_THREADS per field); every warp scans the warp totals itself
+  uint32_t incl[5];
+#pragma unroll
+  for (int f = 0; f < 5; ++f) incl[f] = warp_inclusive_scan(p[f], lane);
+  if (lane == 31)
+#pragma unroll
+    for (int f = 0; f < 5; ++f) tmp[ST_WARPS + 5 * wid + f] = incl[f];
+  __syncthreads();
+  uint32_t ex[5], tot[5];
+#pragma unroll
+  for (int f = 0; f < 5; ++f) {
+    const uint32_t v = lane < ST_WARPS ? tmp[ST_WARPS + 5 * lane + f] : 0u;
+    const uint32_t in = warp_inclusive_scan(v, lane);
+    ex[f] = __shfl_sync(FULL_MASK, in - v, wid) + incl[f] - p[f];
+    tot[f] = __shfl_sync(FULL_MASK, in, ST_WARPS - 1);
+  }
+  auto field = [](uint32_t v, int c) { return (v >> (16 * (c & 1))) & 0xFFFFu; };
+  uint32_t GT = (tot[4] & 0xFFFFu), EQ = (tot[4] >> 16);
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    GT += field(tot[c >> 1], c);
+    EQ += field(tot[2 + (c >> 1)], c);
+  }
+  const uint32_t qq = (uint32_t)q;
+  const uint32_t K = GT + (EQ < qq ? EQ : qq);
+  const uint32_t R0 = K * m / nr, R1 = K * (m + 1) / nr;
+  uint32_t gbase = 0, ebase = 0;
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    if (c < NCH) {
+      uint32_t g0 = gbase + field(ex[c >> 1], c), e0 = ebase + field(ex[2 + (c >> 1)], c);
+      uint32_t bits = gb[c] | eb[c];
+      while (bits) {   // the chunk's channels with key >= T, in order
+        const int h = __ffs(bits) - 1;
+        const uint32_t below = (1u << h) - 1u;
+        const uint32_t g = g0 + (uint32_t)__popc(gb[c] & below), e = e0 + (uint32_t)__popc(eb[c] & below);
+        const bool isg = (gb[c] >> h) & 1u;
+        if (isg || e < qq) {
+          const uint32_t r = g + (e < qq ? e : qq);
+          if (r >= R0 && r < R1) klist[r - R0] = (uint16_t)(8 * (tid + c * ST_THREADS) + h);
+        }
+        bits &= bits - 1;
+      }
+    }
+    gbase += field(tot[c >> 1], c);
+    ebase += field(tot[2 + (c >> 1)], c);
+  }
+  if (tg | te) {
+    const uint32_t g = gbase + (ex[4] & 0xFFFFu), e = ebase + (ex[4] >> 16);
+    if (tg || e < qq) {
+      const uint32_t r = g + (e < qq ? e : qq);
+      if (r >= R0 && r < R1) klist[r - R0] = (uint16_t)jt;
+    }
+  }
+  __syncthreads();
+  return (int)(R1 - R0);
 }
 
 }  // namespace duo

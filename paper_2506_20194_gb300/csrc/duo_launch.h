@@ -46,6 +46,9 @@ struct CmbArgs {
   int thresh;            // in: 1 = threshold mask (keep key > tau_key), 0 = top-k / listed
   uint32_t tau_key;      // in: threshold as an fp16 magnitude bit pattern (bits & 0x7FFF)
   int vbits;             // in: bits of a stored value: 16 (fp16), 8 or 4 (RTN codes)
+  unsigned int* status;  // device status word of the launch (the first handle's):
+                         // bit 0 a bounded wait ran out, bit 1 a bad record or id
+  unsigned long long wait_ns;   // limit of every bounded wait (0: the 1 s default)
   int nruns;             // set by the launcher: > 0 when each (problem, segment)
                          // run has CTAs of its own: run r (items r*k .. r*k+k-1)
                          // goes to CTAs run_cta[r] .. run_cta[r+1]-1
@@ -53,6 +56,7 @@ struct CmbArgs {
 };
 
 struct Idx16Args {
+  unsigned int* status;  // device status word of the launch (the handle's)
   const uint8_t* data;
   const uint64_t* colptr;
   const uint32_t* cnt;
@@ -64,6 +68,14 @@ struct Idx16Args {
   const uint16_t* kidx;
   const uint16_t* kval;
 };
+
+// SM count and opt-in shared memory per block of the current device
+// (cached per device).
+struct DevProps {
+  int nsm = 0;
+  int smem_optin = 0;
+};
+cudaError_t dev_props(DevProps* out);
 
 // spMspV over the bitmask format (fused when a.kidx == nullptr).  Zeroes
 // every y itself (no memset needed before it).
@@ -100,8 +112,9 @@ cudaError_t launch_idx16_scatter(const uint16_t* W, int64_t O, int64_t I, int64_
                                  const uint32_t* cnt_js, const uint32_t* cnt,
                                  const uint64_t* colptr, uint8_t* data, cudaStream_t st);
 
-// Reads and clears the device status word (bit 0: a bounded wait ran out,
-// bit 1: a record size outside the format's bounds).
+// Reads and clears the process-wide device status word of the kernels that
+// run without a handle (the sparsifiers): bit 0 a bounded wait ran out,
+// bit 1 a record size or id outside the format's bounds.
 cudaError_t read_and_clear_status(unsigned int* out);
 
 }  // namespace duo

@@ -5,6 +5,7 @@
 // device status word needs no relocatable device code.
 #include <algorithm>
 #include <cstdio>
+#include <mutex>
 
 #define DUO_STATUS_OWNER
 #include "duo_device.cuh"
@@ -15,17 +16,14 @@ namespace duo {
 // ------------------------------------------------------------------------
 // Device properties (cached per device).
 // ------------------------------------------------------------------------
-struct DevProps {
-  int nsm = 0;
-  int smem_optin = 0;
-};
-
-static cudaError_t dev_props(DevProps* out) {
+cudaError_t dev_props(DevProps* out) {
+  static std::mutex mu;
   static DevProps cache[64];
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lk(mu);
   if (cache[dev].nsm == 0) {
     DevProps p;
     e = cudaDeviceGetAttribute(&p.nsm, cudaDevAttrMultiProcessorCount, dev);
@@ -726,6 +724,11 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   }
   for (int i = tid; i < 2 * SEG_ROWS; i += CMB_THREADS) tile[i] = 0.f;
   if (MODE == CMB_TOPK) select_clear(sel);
+  // x into L2 while the previous kernel finishes: a prefetch reads nothing
+  // into this CTA, and L2 is coherent, so a later write to x by that kernel
+  // is what the loads after the wait see.
+  if (FUSED && tid < (2 * a.I + 127) / 128)
+    prefetch_line_l2(reinterpret_cast<const uint8_t*>(a.x) + 128 * tid);
   // Inputs, y and the grid barrier words may be the previous kernel's.
   griddep_wait();
   // Generation of the grid barrier before this CTA arrives on it (read here,
@@ -735,18 +738,24 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   if (tid == 0) {
     gen0 = ld_relaxed_gpu(a.bar + 1);
   }
-  if (FUSED) load_x_to_smem(xs, a.x, a.I);
+  // Fused modes: x and the selection straight from registers when x fits
+  // (select_window), else through shared memory.
+  const bool regs = FUSED && select_window_ok<CMB_THREADS>(a.x, a.I);
+  if (FUSED && !regs) load_x_to_smem(xs, a.x, a.I);
   uint32_t u0, u1;   // this CTA's items (32-bit: the launcher keeps counts < 2^31)
   int r0 = 0;        // kept rank of its first item
   int pr = 0, sr = 0, c0 = 0, c1 = 0;   // fused modes: run (product, segment), channel range
+  uint32_t rm = 0, rn = 1;               // fused modes: this CTA's index in its run, the run's CTAs
   if (FUSED) {
-    // Run r (product pr, segment sr) is split into channel ranges; items are
-    // the kept channels of this CTA's range, numbered from 0.
+    // Run r (product pr, segment sr): every CTA of it takes an equal share
+    // of the run's kept channels in index order (select_window), or, on the
+    // shared-memory path, the kept channels of its own channel range.
     int r = 0;
     while (r + 1 < a.nruns && (unsigned)a.run_cta[r + 1] <= blockIdx.x) ++r;
-    const uint32_t n = a.run_cta[r + 1] - a.run_cta[r], m = blockIdx.x - a.run_cta[r];
-    c0 = (int)((uint32_t)a.I * m / n);
-    c1 = (int)((uint32_t)a.I * (m + 1) / n);
+    rn = a.run_cta[r + 1] - a.run_cta[r];
+    rm = blockIdx.x - a.run_cta[r];
+    c0 = (int)((uint32_t)a.I * rm / rn);
+    c1 = (int)((uint32_t)a.I * (rm + 1) / rn);
     sr = r;
     while (pr < a.np - 1 && sr >= a.p[pr].S) sr -= a.p[pr++].S;
     u0 = u1 = 0;
@@ -765,7 +774,17 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     u1 = (uint32_t)((uint64_t)total * (blockIdx.x + 1) / gridDim.x);
   }
   __syncthreads();
-  if (FUSED) {
+  if (FUSED && regs) {
+    constexpr bool TK = MODE == CMB_TOPK;
+    const int nch = ((a.I >> 3) + CMB_THREADS - 1) / CMB_THREADS;
+    const int tk = (int)a.tau_key;
+    int nw;
+    if (nch <= 1) nw = select_window<TK, 1, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, rm, rn, klist, sel->tmp);
+    else if (nch == 2) nw = select_window<TK, 2, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, rm, rn, klist, sel->tmp);
+    else if (nch == 3) nw = select_window<TK, 3, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, rm, rn, klist, sel->tmp);
+    else nw = select_window<TK, 4, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, rm, rn, klist, sel->tmp);
+    u1 = (uint32_t)nw;
+  } else if (FUSED) {
     // The kept set as a threshold (top-k: computed here; threshold mask:
     // given), then this CTA's kept channels of its range, numbered from 0.
     int T = (int)a.tau_key, cut = -1;
@@ -812,7 +831,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     const uint32_t* qsrc = nullptr;
     if (QUANT) {
       const ItemCursor ci = cursor_at(u0);   // a CTA of a coded launch serves one run
-      gA = FUSED ? c0 / QGROUP : __shfl_sync(FULL_MASK, q[0].g, 0);
+      gA = FUSED ? (nv > 0 ? klist[0] / QGROUP : 0) : __shfl_sync(FULL_MASK, q[0].g, 0);
       const CmbProb& P = a.p[ci.p];
       qsrc = P.qtab + ((size_t)ci.s * P.G + gA) * SEG_ROWS;
     }
@@ -830,7 +849,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
           if (v >= nv) continue;
           const Resolved r = q[d];
           if (r.bad(slot_bytes)) {
-            atomicOr(&g_status, STATUS_FORMAT);
+            atomicOr(a.status, STATUS_FORMAT);
             abort_flag = 1;
             stop = true;
             continue;
@@ -842,7 +861,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
           // Fill n of a slot waits until fill n - 1 has been consumed.  Fill
           // n - 1 was issued in an earlier round (nslot >= 32), after fill
           // n - 2 had been released, so the "empty" phase parity is exact.
-          if (sc.n > 0 && !mbar_wait_bounded(&empty[sc.slot], (uint32_t)((sc.n - 1) & 1), &abort_flag)) {
+          if (sc.n > 0 && !mbar_wait_bounded(&empty[sc.slot], (uint32_t)((sc.n - 1) & 1), &abort_flag, a.status, a.wait_ns)) {
             stop = true;
             continue;
           }
@@ -858,7 +877,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
           int seq = 0;
           if (pend) {
             if (r.bad(slot_bytes)) {
-              atomicOr(&g_status, STATUS_FORMAT);
+              atomicOr(a.status, STATUS_FORMAT);
               abort_flag = 1;
               stop = true;
               pend = false;
@@ -873,7 +892,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
           // prefix of the warp); a kept list out of group order is rejected.
           const int prev = __shfl_up_sync(FULL_MASK, seq, 1);
           if (pend && (seq < 0 || seq < (lane == 0 ? last_seq : prev))) {
-            atomicOr(&g_status, STATUS_FORMAT);
+            atomicOr(a.status, STATUS_FORMAT);
             abort_flag = 1;
             stop = true;
             pend = false;
@@ -882,7 +901,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
           while (true) {
             if (pend && seq < tarm) {   // table armed: issue
               if (sc.n > 0 &&
-                  !mbar_wait_bounded(&empty[sc.slot], (uint32_t)((sc.n - 1) & 1), &abort_flag)) {
+                  !mbar_wait_bounded(&empty[sc.slot], (uint32_t)((sc.n - 1) & 1), &abort_flag, a.status, a.wait_ns)) {
                 stop = true;
               } else {
                 xval[sc.slot] = (uint32_t)r.xb | ((uint32_t)seq << 16);
@@ -902,7 +921,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
             bool ok = true;
             if (tarm >= QNTB) {
               // Its buffer's previous load (table tarm - QNTB) has landed ...
-              if (lane == 0) ok = mbar_wait_bounded(&tfull[b], (uint32_t)((tarm / QNTB - 1) & 1), &abort_flag);
+              if (lane == 0) ok = mbar_wait_bounded(&tfull[b], (uint32_t)((tarm / QNTB - 1) & 1), &abort_flag, a.status, a.wait_ns);
               ok = __shfl_sync(FULL_MASK, ok, 0);
               // ... and every item before the first of table tarm - QNTB + 1
               // is released: lane c checks consumer c's count.
@@ -911,10 +930,10 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
               const int* cw = &cons[lane < CMB_NC ? lane : 0];
               const uint64_t t0 = globaltimer_ns();
               while (ok && !__all_sync(FULL_MASK, ld_acquire_cta_shared(cw) >= need)) {
-                const bool late = globaltimer_ns() - t0 > WAIT_LIMIT_NS;
+                const bool late = globaltimer_ns() - t0 > a.wait_ns;
                 if (__any_sync(FULL_MASK, late || abort_flag != 0)) {
                   if (lane == 0 && late) {
-                    atomicOr(&g_status, STATUS_TIMEOUT);
+                    atomicOr(a.status, STATUS_TIMEOUT);
                     abort_flag = 1;
                   }
                   ok = false;
@@ -946,8 +965,8 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       const uint64_t t0 = globaltimer_ns();
       while (ld_acquire_gpu(a.bar + 1) == gen0) {
         __nanosleep(64);
-        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
-          atomicOr(&g_status, STATUS_TIMEOUT);
+        if (globaltimer_ns() - t0 > a.wait_ns) {
+          atomicOr(a.status, STATUS_TIMEOUT);
           abort_flag = 1;
           break;
         }
@@ -959,14 +978,14 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       for (int v = last_v; v >= 0 && v > last_v - nslot; v -= 32) {
         SlotCursor w;
         w.set(v, nslot);
-        mbar_wait_limited(&full[w.slot], (uint32_t)(w.n & 1));
+        mbar_wait_limited(&full[w.slot], (uint32_t)(w.n & 1), a.status, a.wait_ns);
       }
     }
     if (QUANT && lane == 0) {
       // A table no consumer waited on (a group without kept channels) may
       // still be landing: wait for the last QNTB before the CTA exits.
       for (int t = tarm > QNTB ? tarm - QNTB : 0; t < tarm; ++t)
-        mbar_wait_limited(&tfull[t % QNTB], (uint32_t)((t / QNTB) & 1));
+        mbar_wait_limited(&tfull[t % QNTB], (uint32_t)((t / QNTB) & 1), a.status, a.wait_ns);
     }
   } else {
     // ---------------- consumers ----------------
@@ -1004,7 +1023,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     // (group * CMB_NC <= nslot): when it waits for fill n, fill n - 1 is
     // consumed and fill n + 1 not yet issued, so the "full" parity is exact.
     auto wait_item = [&](const SlotCursor& q) -> bool {
-      return mbar_wait_bounded(&full[q.slot], (uint32_t)(q.n & 1), &abort_flag);
+      return mbar_wait_bounded(&full[q.slot], (uint32_t)(q.n & 1), &abort_flag, a.status, a.wait_ns);
     };
     auto release = [&](const SlotCursor& q) { mbar_arrive(&empty[q.slot]); };
     // Coded formats: the grid table of an item's group (its table number is
@@ -1014,7 +1033,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     const uint32_t* tcur = nullptr;
     auto table_for = [&](uint32_t seq) -> const uint32_t* {
       if ((int)seq != cur_seq) {
-        if (!mbar_wait_bounded(&tfull[seq % QNTB], (seq / QNTB) & 1u, &abort_flag)) return nullptr;
+        if (!mbar_wait_bounded(&tfull[seq % QNTB], (seq / QNTB) & 1u, &abort_flag, a.status, a.wait_ns)) return nullptr;
         cur_seq = (int)seq;
         tcur = qt + (size_t)(seq % QNTB) * SEG_ROWS + lane;
       }
@@ -1125,8 +1144,8 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
         while (ld_acquire_gpu(a.bar + 1) == gen0c) {
           if (ld_acquire_cta_shared(&grid_open) == 1) return;
           __nanosleep(64);
-          if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
-            atomicOr(&g_status, STATUS_TIMEOUT);
+          if (globaltimer_ns() - t0 > a.wait_ns) {
+            atomicOr(a.status, STATUS_TIMEOUT);
             abort_flag = 1;
             return;
           }
@@ -1198,6 +1217,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
 
 cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   CmbArgs a = a0;
+  if (a.wait_ns == 0) a.wait_ns = WAIT_LIMIT_NS;
   DevProps dp;
   cudaError_t e = dev_props(&dp);
   if (e != cudaSuccess) return e;
@@ -1344,7 +1364,7 @@ __global__ void __launch_bounds__(IDX16_THREADS, 1) idx16_spmspv_kernel(const Id
       xb = __ldg(a.kval + i);
     }
     if (j >= a.I) {
-      if (lane == 0) atomicOr(&g_status, STATUS_FORMAT);
+      if (lane == 0) atomicOr(a.status, STATUS_FORMAT);
       continue;
     }
     const uint32_t n = __ldg(a.cnt + j);

@@ -69,6 +69,9 @@ def load_library(path: str | None = None):
     lib.duo_packed_export.argtypes = [vp, i32, vp, i64]
     lib.duo_pack_cmb_noalloc.argtypes = [vp, i64, i64, i64, vp, vp, i64, ctypes.POINTER(i64), vp]
     lib.duo_device_status.argtypes = [vp]
+    lib.duo_packed_status.argtypes = [vp, vp]
+    # internal, for the failure-detection test (not part of include/duo.h)
+    lib.duo_test_spmspv_blocked.argtypes = [vp, vp, i64, vp, ctypes.c_uint64, vp]
     lib.duo_copy.argtypes = [vp, vp, i64, vp]
     lib.duo_calib_create.argtypes = [i64, i64, vp, ctypes.POINTER(vp)]
     lib.duo_calib_precompute.argtypes = [vp, vp, i64, ctypes.c_float, i32, vp]
@@ -85,7 +88,8 @@ def load_library(path: str | None = None):
                  "duo_packed_query", "duo_packed_export", "duo_device_status", "duo_abi_version",
                  "duo_pack_cmb_noalloc", "duo_sparsify_threshold", "duo_spmspv_threshold",
                  "duo_calib_create", "duo_calib_precompute", "duo_calib_status", "duo_calib_export",
-                 "duo_calib_score", "duo_calib_free", "duo_calib_prune", "duo_copy", "duo_calib_query"):
+                 "duo_calib_score", "duo_calib_free", "duo_calib_prune", "duo_copy", "duo_calib_query",
+                 "duo_packed_status", "duo_test_spmspv_blocked"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -254,6 +258,11 @@ def duo_free(h: Packed):
 
 def duo_device_status(stream=None) -> int:
     return load_library().duo_device_status(_stream_ptr(stream))
+
+
+def duo_packed_status(h: Packed, stream=None) -> int:
+    """Status of the launches whose first handle is h (read and cleared)."""
+    return load_library().duo_packed_status(h.handle, _stream_ptr(stream))
 
 
 def duo_copy(dst: torch.Tensor, src: torch.Tensor, stream=None):
