@@ -21,8 +21,10 @@
  * original channel perm[p]).
  *
  * Precision: X is fp16; H and dX X_hat^T are fp16 products accumulated in
- * fp32; the factorisation and the products with L are fp32.  The act_order
- * permutation is decided on exact integer sums, so it is reproducible.
+ * fp32; the factorisation and the products with L are fp32 (on the tensor
+ * cores: each fp32 operand split into three bf16 pieces, six piece products
+ * summed in fp32).  The act_order permutation is decided on exact integer
+ * sums, so it is reproducible.
  *
  * All pointers named *_dev are device memory.  Calls are asynchronous on the
  * given stream (a cudaStream_t passed as void*) unless stated.
@@ -45,8 +47,12 @@ typedef struct duo_calib duo_calib;
 
 /*
  * duo_calib_create -- allocates a context for k channels and m tokens:
- * cuBLAS / cuSOLVER handles bound to `stream` and about 9 k^2 fp32 plus
- * 2 k m fp16 of device memory.  Synchronous.
+ * about 9 k^2 fp32 plus 2 k m fp16 of device memory, two buffers for
+ * prepared tensor-core operands (k^2 fp32 split into three bf16 pieces,
+ * 6 k^2 bytes each, at least), and a high-priority side stream with two
+ * events, on which the factorisation runs its diagonal blocks (work
+ * enqueued on the caller's stream forks to it and joins back, so a stream
+ * capture takes it in).  Synchronous.
  *   k : 1..32768 channels.   m : 1..2^20 tokens.
  * Errors: DUO_EINVAL (sizes, NULL), DUO_ENOMEM, DUO_ECUDA.
  */
@@ -70,7 +76,10 @@ int duo_calib_precompute(duo_calib* h, const void* X_fp16_dev, int64_t keep, flo
 
 /* Synchronises `stream`, then reports the last precompute's factorisation:
  * DUO_OK, or DUO_ERANGE if the Cholesky factorisation of the dampened H
- * failed (not positive definite); DUO_ECUDA on a CUDA error. */
+ * failed (not positive definite); DUO_ETIMEOUT if a bounded wait inside a
+ * tensor-core product ran out since the last call (a process-wide word,
+ * read and cleared here; that product's output tile was not written);
+ * DUO_ECUDA on a CUDA error. */
 int duo_calib_status(const duo_calib* h, void* stream);
 
 /* Buffers of a context (device pointers owned by the context; valid until

@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT = os.path.join(PKG, "libduo.so")
 BUILD_DIR = os.path.join(PKG, "_build")
-SOURCES = ("kernels.cu", "api.cu", "noalloc.cu", "calib.cu", "copy.cu")
+SOURCES = ("kernels.cu", "api.cu", "noalloc.cu", "calib.cu", "copy.cu", "tcgemm.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -55,11 +55,7 @@ def build_library(verbose_ptxas: bool = False, force: bool = False) -> str:
     with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(lambda s: _compile(s, extra), SOURCES))
     tmp = OUT + ".tmp"
-    # cuBLAS and cuSOLVER (the calibration precompute's GEMMs and
-    # factorisation) are the toolkit's shared libraries, found through rpath.
-    cuda_lib = os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(nvcc_path()))), "lib64")
-    cmd = [nvcc_path(), *ARCH, "-shared", "-o", tmp, *objs, "-lcublas", "-lcusolver", "-lcudart_static",
-           "-lrt", "-ldl", "-lpthread", "-Xlinker", f"-rpath={cuda_lib}"]
+    cmd = [nvcc_path(), *ARCH, "-shared", "-o", tmp, *objs, "-lcudart_static", "-lrt", "-ldl", "-lpthread"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

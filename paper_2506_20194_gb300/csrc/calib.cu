@@ -2,22 +2,28 @@
 // per-token sparse input, the Hessian and its inverse-Cholesky factor, Q, U,
 // a, b, c, D and the efficient pruning score (C ABI: include/duo_calib.h).
 //
-// Plain GEMMs go to cuBLAS: H = X_hat X_hat^T and dX X_hat^T with fp16
-// inputs and fp32 accumulation on the tensor cores, the products with L in
-// fp32 (emulated with bf16 tensor-core products, see kL_COMPUTE).  The
-// factorisation goes to cuSOLVER.  Everything else is a kernel here.
+// Every dense contraction runs on the tcgen05 GEMM of tcgemm.cu: H = X_hat
+// X_hat^T and dX X_hat^T with fp16 operands (exact products, fp32 sums), the
+// products with L, the factorisation's panels and updates, the triangular
+// inverse and the sweep's lazy batch update with fp32 operands (three bf16
+// pieces each, six piece products: fp32-level results).  Everything else is
+// a kernel here.
 //
 // L (lower, H^-1 = L L^T) comes from one Cholesky factorisation and one
 // triangular inverse: with J the index reversal, factor J H J = C C^T; then
 // H^-1 = J C^-T C^-1 J = (J C^-T J)(J C^-T J)^T and J C^-T J is lower with a
 // positive diagonal, so it is L.  (Forming H^-1 and factoring it again would
-// take twice the flops.)  The triangular inverse is computed here by
+// take twice the flops.)  The factorisation is blocked and right-looking
+// with 128-column blocks: one CTA factors a diagonal block C11 and inverts
+// it in the same elimination (the row operations that reduce the block to
+// C11^T turn the identity into C11^-1), the panel below is A21 C11^-T on the
+// tensor cores, and the trailing matrix takes the rank-128 update
+// -L21 L21^T (lower tiles only).  The triangular inverse is computed by
 // recursive doubling: 64 x 64 diagonal blocks are inverted in shared memory,
 // then for s = 64, 128, ... each pair [A 0; B D] of s x s diagonal blocks
-// gets its off-diagonal block -D^-1 B A^-1 from two batched tensor-core
-// GEMMs.  (cuSOLVER's trtri took 8.3 ms at k = 4096 on GB300, its
-// factorisation 2.1 ms.)  C is kept in a kp x kp buffer, kp = 64 * 2^j >= k,
-// whose trailing diagonal block is the identity.
+// gets its off-diagonal block -D^-1 B A^-1 from two batched GEMMs.  C is kept
+// in a kp x kp buffer, kp = 64 * 2^j >= k, whose trailing diagonal block is
+// the identity.
 #include <cstdint>
 #include <cstdlib>
 #include <cstring>
@@ -25,12 +31,11 @@
 #include <new>
 #include <unordered_set>
 
-#include <cublas_v2.h>
 #include <cuda_runtime.h>
-#include <cusolverDn.h>
 
 #include "duo_calib.h"
 #include "duo_device.cuh"
+#include "tcgemm.h"
 
 namespace duo {
 namespace calib {
@@ -47,11 +52,6 @@ inline int64_t tri_pad(int64_t k) {
   while (kp < k) kp *= 2;
   return kp;
 }
-// Products with L in fp32 through cuBLAS's BF16x9 emulation on the tensor
-// cores: measured on GB300 at k = 4096, 215 TFLOP/s with a max error of
-// 7e-7 relative, against 67 TFLOP/s and 2.5e-6 for the plain fp32 path.
-constexpr cublasComputeType_t kL_COMPUTE = CUBLAS_COMPUTE_32F_EMULATED_16BFX9;
-
 __host__ __device__ inline size_t tok_xs_bytes(int k) { return (2 * (size_t)k + 63) / 64 * 64; }
 
 // X_hat and dX rows of one token (§3: keep the `keep` largest |x|, ties to
@@ -141,29 +141,40 @@ __device__ __forceinline__ bool key_before(U128 a, int ia, U128 b, int ib) {   /
 }
 
 // act_order: perm[rank(i)] = i, rank = channels sorting before i (largest
-// diagonal first, ties to the lower index).  One thread per channel, keys
-// streamed through shared memory.
-__global__ void __launch_bounds__(RANK_THREADS) rank_kernel(const uint64_t* __restrict__ key_hi,
-                                                            const uint64_t* __restrict__ key_lo, int k,
-                                                            int act_order, int* __restrict__ perm) {
+// diagonal first, ties to the lower index).  rank_count_kernel: one thread
+// per channel i, CTA y of RANK_SPLIT compares i with the channels of its
+// slice of j (keys streamed through shared memory) and adds its count to
+// rank[i] (zeroed beforehand); rank_place_kernel scatters.
+constexpr int RANK_SPLIT = 16;
+
+__global__ void __launch_bounds__(RANK_THREADS) rank_count_kernel(const uint64_t* __restrict__ key_hi,
+                                                                  const uint64_t* __restrict__ key_lo, int k,
+                                                                  int* __restrict__ rank) {
   __shared__ uint64_t th[RANK_THREADS], tl[RANK_THREADS];
   const int i = blockIdx.x * RANK_THREADS + threadIdx.x;
   const U128 ki = i < k ? eff_key(key_hi, key_lo, i) : U128{0, 0};
-  int rank = 0;
-  for (int j0 = 0; j0 < k; j0 += RANK_THREADS) {
+  const int per = (k + RANK_SPLIT - 1) / RANK_SPLIT;
+  const int jb = blockIdx.y * per, je = min(k, jb + per);
+  int cnt = 0;
+  for (int j0 = jb; j0 < je; j0 += RANK_THREADS) {
     __syncthreads();
     const int j = j0 + threadIdx.x;
-    if (j < k) {
+    if (j < je) {
       const U128 kj = eff_key(key_hi, key_lo, j);
       th[threadIdx.x] = kj.hi;
       tl[threadIdx.x] = kj.lo;
     }
     __syncthreads();
-    const int n = min(RANK_THREADS, k - j0);
-    if (i < k && act_order)
-      for (int q = 0; q < n; ++q) rank += key_before(U128{th[q], tl[q]}, j0 + q, ki, i) ? 1 : 0;
+    const int n = min(RANK_THREADS, je - j0);
+    if (i < k)
+      for (int q = 0; q < n; ++q) cnt += key_before(U128{th[q], tl[q]}, j0 + q, ki, i) ? 1 : 0;
   }
-  if (i < k) perm[act_order ? rank : i] = i;
+  if (i < k && cnt > 0) atomicAdd(rank + i, cnt);
+}
+
+__global__ void rank_place_kernel(const int* __restrict__ rank, int k, int act_order, int* __restrict__ perm) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < k) perm[act_order ? rank[i] : i] = i;
 }
 
 // damp * mean(diag(H)) from the exact keys (one block).
@@ -185,9 +196,10 @@ __global__ void damp_kernel(const uint64_t* __restrict__ key_hi, const uint64_t*
 }
 
 // Reordered, dampened H (row-major Hp, and its index reversal Hr for the
-// factorisation) and reordered G = dX X_hat^T (row-major Gp).  H and G are
-// cuBLAS column-major: G[i + j k] = (dX X_hat^T)_ij.
-__global__ void gather_kernel(const float* __restrict__ H, const float* __restrict__ G,
+// factorisation) and reordered G = dX X_hat^T (row-major Gp).  H (symmetric)
+// and GT hold H_ij and G_ij at [j + i k], so output row p reads the one
+// contiguous column perm[p] of each (16 KB at k = 4096) in permuted order.
+__global__ void gather_kernel(const float* __restrict__ H, const float* __restrict__ GT,
                               const int* __restrict__ perm, const uint64_t* __restrict__ key_hi,
                               const uint64_t* __restrict__ key_lo, int k, int kp,
                               const float* __restrict__ dampadd, float* __restrict__ Hp,
@@ -196,14 +208,14 @@ __global__ void gather_kernel(const float* __restrict__ H, const float* __restri
   const int p = blockIdx.y;
   if (q >= k) return;
   const int op = perm[p], oq = perm[q];
-  float h = H[(size_t)op + (size_t)oq * k];
+  float h = H[(size_t)oq + (size_t)op * k];
   if (p == q) {
     if (key_hi[op] == 0 && key_lo[op] == 0) h = 1.f;
     h += *dampadd;
   }
   Hp[(size_t)p * k + q] = h;
   Hr[(size_t)(k - 1 - p) * kp + (k - 1 - q)] = h;
-  Gp[(size_t)p * k + q] = G[(size_t)op + (size_t)oq * k];
+  Gp[(size_t)p * k + q] = GT[(size_t)oq + (size_t)op * k];
 }
 
 // L (row-major) from C^-1 (column-major, lower, leading dimension kp):
@@ -254,6 +266,236 @@ __global__ void __launch_bounds__(TRI_BASE) tri_base_inverse_kernel(float* __res
   }
   __syncthreads();
   for (int c = 0; c < TRI_BASE; ++c) blk[t + (size_t)c * ld] = x[t][c];
+}
+
+// ---- blocked Cholesky factorisation ----
+
+constexpr int CHOL_NB = 128;                 // columns per block
+constexpr int CHOL_SUB = 32;                 // columns per sub-block (one warp)
+constexpr int CHOL_THREADS = 256;
+constexpr int CHOL_P = CHOL_NB + 1;          // pitch of the shared 128 x 128 arrays
+constexpr int CHOL_SMEM = (2 * CHOL_NB * CHOL_P + 3 * CHOL_SUB) * (int)sizeof(float);
+
+// The warp's factorisation of the 32 x 32 block F (pitch fp, lower
+// triangle read, factor written in place).  Lane j holds column j of the
+// Schur complement in a.  Step c: lane c publishes its column in shared
+// memory (cbuf, two buffers), every lane reads it back with eight 16-byte
+// broadcast loads, l_ic = a_ic / sqrt(a_cc), lane j >= c writes l_jc to
+// F[j][c], and lanes j > c take a_ij -= l_ic l_jc over all 32 rows (rows
+// above j are not used).  1 / l_cc goes to rdiag[c].  Returns the first
+// pivot (1-based) that was not positive and finite, 0 if none; such a pivot
+// is taken as 1.
+__device__ __forceinline__ int chol_warp_factor(float* F, int fp, float* rdiag, float* cbuf, int lane) {
+  float a[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) a[i] = i >= lane ? F[i * fp + lane] : 0.f;
+  int bad = 0;
+#pragma unroll 1
+  for (int c = 0; c < 32; ++c) {
+    float4* cb = reinterpret_cast<float4*>(cbuf + 32 * (c & 1));
+    if (lane == c) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) cb[q] = make_float4(a[4 * q], a[4 * q + 1], a[4 * q + 2], a[4 * q + 3]);
+    }
+    __syncwarp();
+    float v[32];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float4 t = cb[q];
+      v[4 * q] = t.x;
+      v[4 * q + 1] = t.y;
+      v[4 * q + 2] = t.z;
+      v[4 * q + 3] = t.w;
+    }
+    const float* cs = cbuf + 32 * (c & 1);
+    float p = cs[c];
+    if (!(p > 0.f) || !(p < INFINITY)) {   // warp-uniform
+      if (bad == 0) bad = c + 1;
+      p = 1.f;
+    }
+    const float inv = rsqrtf(p);
+    const float lj = lane == c ? p * inv : cs[lane] * inv;   // l_(lane)c
+    if (lane >= c) F[lane * fp + c] = lj;
+    if (lane == c) rdiag[c] = inv;   // 1 / l_cc
+    if (lane > c) {
+      const float w = lj * inv;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) a[i] = fmaf(-v[i], w, a[i]);
+    }
+  }
+  return bad;
+}
+
+// Forward substitution with the 32 x 32 lower factor F (pitch fp, reciprocal
+// diagonal rd): v <- F^-1 v, in registers (every index a constant).
+__device__ __forceinline__ void chol_forward(float (&v)[32], const float* F, int fp, const float* rd) {
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    float s0 = v[j], s1 = 0.f, s2 = 0.f, s3 = 0.f;   // four chains against the FMA latency
+#pragma unroll
+    for (int t = 0; t < j; t += 4) {
+      s0 = fmaf(-F[j * fp + t], v[t], s0);
+      if (t + 1 < j) s1 = fmaf(-F[j * fp + t + 1], v[t + 1], s1);
+      if (t + 2 < j) s2 = fmaf(-F[j * fp + t + 2], v[t + 2], s2);
+      if (t + 3 < j) s3 = fmaf(-F[j * fp + t + 3], v[t + 3], s3);
+    }
+    v[j] = ((s0 + s1) + (s2 + s3)) * rd[j];
+  }
+}
+
+// Factor of one diagonal block and its inverse.  The block is E(j0 + i,
+// j0 + j), i, j < b <= 128, of the column-major buffer E (leading dimension
+// kp), lower triangle read; it holds the Schur complement left by the
+// earlier blocks (the identity stands in beyond b).  Writes C11 (lower,
+// zeros above the diagonal) back in place and X = C11^-1 to Linv (row-major
+// 128 x 128, the identity beyond b).
+//
+// Four sub-blocks of 32 columns, o = 0, 32, 64, 96, each in three phases
+// separated by barriers:
+//  1. warp 0 factors the 32 x 32 diagonal sub-block, D = C_ss C_ss^T
+//     (chol_warp_factor).
+//  2. one forward substitution with C_ss per thread (128 threads): each
+//     panel row below, L_is^T = C_ss^-1 A_is^T; each of the o columns of X
+//     already started on rows o .. o+31, X_s = C_ss^-1 X_s (the row
+//     operations of this sub-block applied to what the earlier ones left);
+//     and the 32 columns of C_ss^-1 itself (X's diagonal sub-block).
+//  3. the rank-32 updates of everything below, in 4 x 4 register tiles: the
+//     trailing block A_ij -= L_is L_js^T (lower tiles), and X_i -= L_is X_s
+//     on rows i >= o + 32 (columns < o + 32; right of those X is still 0).
+// Rows of X above the current sub-block are final once their sub-block is
+// done: X = C11^-1 is the elimination's row operations applied to I.  A
+// pivot that is not positive and finite marks info (first column, 1-based,
+// as a Cholesky routine reports it) and is replaced by 1.
+__global__ void __launch_bounds__(CHOL_THREADS, 1) chol_diag_kernel(float* __restrict__ E, int kp, int j0, int b,
+                                                                 float* __restrict__ Linv,
+                                                                 int* __restrict__ info) {
+  extern __shared__ float csm[];
+  float* A = csm;                               // [128][CHOL_P]: the block, then C11 (lower)
+  float* X = csm + CHOL_NB * CHOL_P;            // [128][CHOL_P]: C11^-1 (lower)
+  float* rd = X + CHOL_NB * CHOL_P;             // [32]: 1 / diagonal of the current C_ss
+  float* cbuf = rd + CHOL_SUB;                  // [2][32]: the warp factor's broadcast column
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  float* blk = E + (size_t)j0 * ((size_t)kp + 1);
+  // the block in batches of 32 independent loads per thread (a loop that
+  // stored each load before issuing the next would pay the memory latency
+  // on every element)
+  constexpr int LOAD_BATCH = 32;
+#pragma unroll 1
+  for (int base = 0; base < CHOL_NB * CHOL_NB; base += LOAD_BATCH * CHOL_THREADS) {
+    float v[LOAD_BATCH];
+#pragma unroll
+    for (int u = 0; u < LOAD_BATCH; ++u) {
+      const int idx = base + u * CHOL_THREADS + tid;
+      const int i = idx & (CHOL_NB - 1), j = idx >> 7;   // i fastest: E is column-major
+      v[u] = (i < b && j < b) ? (i >= j ? __ldg(blk + i + (size_t)j * kp) : 0.f) : (i == j ? 1.f : 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < LOAD_BATCH; ++u) {
+      const int idx = base + u * CHOL_THREADS + tid;
+      const int i = idx & (CHOL_NB - 1), j = idx >> 7;
+      A[i * CHOL_P + j] = v[u];
+      X[i * CHOL_P + j] = 0.f;
+    }
+  }
+  __syncthreads();
+  for (int o = 0; o < CHOL_NB; o += CHOL_SUB) {
+    float* F = A + o * CHOL_P + o;              // the sub-block's factor, pitch CHOL_P
+    // ---- 1. factor the diagonal sub-block (warp 0) ----
+    if (warp == 0) {
+      const int bad = chol_warp_factor(F, CHOL_P, rd, cbuf, lane);
+      if (lane == 0 && bad > 0 && o + bad - 1 < b) atomicCAS(info, 0, j0 + o + bad);
+    }
+    __syncthreads();
+    // ---- 2. forward substitutions: panel rows, columns of X ----
+    const int below = CHOL_NB - o - CHOL_SUB;   // rows under the sub-block
+    if (tid < CHOL_NB) {                         // below + o + 32 == 128 solves
+      float v[CHOL_SUB];
+      if (tid < below) {                         // panel row o + 32 + tid
+        const float* ar = A + (o + CHOL_SUB + tid) * CHOL_P + o;
+#pragma unroll
+        for (int t = 0; t < CHOL_SUB; ++t) v[t] = ar[t];
+      } else if (tid < below + o) {              // column c < o of X's rows o .. o+31
+        const int c = tid - below;
+#pragma unroll
+        for (int t = 0; t < CHOL_SUB; ++t) v[t] = X[(o + t) * CHOL_P + c];
+      } else {                                   // column q of the identity
+        const int q = tid - below - o;
+#pragma unroll
+        for (int t = 0; t < CHOL_SUB; ++t) v[t] = t == q ? 1.f : 0.f;
+      }
+      chol_forward(v, F, CHOL_P, rd);
+      if (tid < below) {
+        float* ar = A + (o + CHOL_SUB + tid) * CHOL_P + o;
+#pragma unroll
+        for (int t = 0; t < CHOL_SUB; ++t) ar[t] = v[t];
+      } else {
+        const int c = tid - below;               // o + q for the identity columns
+#pragma unroll
+        for (int t = 0; t < CHOL_SUB; ++t) X[(o + t) * CHOL_P + c] = v[t];
+      }
+    }
+    __syncthreads();
+    if (below == 0) break;
+    // ---- 3. rank-32 updates below, in 4 x 4 tiles ----
+    const int nrt = below / 4;                        // row tiles
+    const int xct = (o + CHOL_SUB) / 4;               // X column tiles
+    const int nx = nrt * xct, ntask = nx + nrt * (nrt + 1) / 2;
+    for (int task = tid; task < ntask; task += CHOL_THREADS) {
+      int i0, c0;
+      const float* Y;                                 // Y(t, c): X[o + t][c] or A[c][o + t]
+      int ys_t, ys_c;
+      float* out;
+      if (task < nx) {
+        i0 = o + CHOL_SUB + 4 * (task / xct);
+        c0 = 4 * (task % xct);
+        Y = X + o * CHOL_P;
+        ys_t = CHOL_P;
+        ys_c = 1;
+        out = X;
+      } else {
+        int tt = task - nx, ti = 0;                   // lower tile (ti, tj), tj <= ti
+        while (tt > ti) {
+          tt -= ti + 1;
+          ++ti;
+        }
+        i0 = o + CHOL_SUB + 4 * ti;
+        c0 = o + CHOL_SUB + 4 * tt;
+        Y = A + o;
+        ys_t = 1;
+        ys_c = CHOL_P;
+        out = A;
+      }
+      float acc[4][4] = {};
+      const float* Lr = A + i0 * CHOL_P + o;
+#pragma unroll 4
+      for (int t = 0; t < CHOL_SUB; ++t) {
+        float lv[4], yv[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          lv[e] = Lr[e * CHOL_P + t];
+          yv[e] = Y[t * ys_t + (c0 + e) * ys_c];
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+#pragma unroll
+          for (int f = 0; f < 4; ++f) acc[e][f] = fmaf(lv[e], yv[f], acc[e][f]);
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+#pragma unroll
+        for (int f = 0; f < 4; ++f) out[(i0 + e) * CHOL_P + c0 + f] -= acc[e][f];
+    }
+    __syncthreads();
+  }
+  // C11 back into E (column-major, zeros above the diagonal), X to Linv
+  for (int idx = tid; idx < CHOL_NB * CHOL_NB; idx += CHOL_THREADS) {
+    const int i = idx & (CHOL_NB - 1), j = idx >> 7;
+    if (i < b && j < b) blk[i + (size_t)j * kp] = i >= j ? A[i * CHOL_P + j] : 0.f;
+  }
+  for (int idx = tid; idx < CHOL_NB * CHOL_NB; idx += CHOL_THREADS) {
+    const int i = idx >> 7, j = idx & (CHOL_NB - 1);   // j fastest: Linv is row-major
+    Linv[idx] = j <= i ? X[i * CHOL_P + j] : 0.f;
+  }
 }
 
 // Row p of Q (row-major): U = its part right of the diagonal, b_p = |U_p|^2,
@@ -658,19 +900,18 @@ struct duo_calib {
   uint32_t magic;
   int device;
   int64_t k, m, kp;   // kp: padded order of the triangular factor
-  cublasHandle_t blas;
-  cusolverDnHandle_t solver;
-  cusolverDnParams_t params;
   uint16_t *Xh, *dX;
   float *H, *G, *Hp, *Hr, *L, *Gp, *Q, *U, *D;
   float *a_orig, *a, *b, *c, *col, *dampadd;
   uint64_t *key_hi, *key_lo;
   int* perm;
+  int* rank;   // act_order ranks (scratch)
   int* info;   // factorisation status
-  void* dwork;
-  size_t dwork_bytes;
-  void* hwork;
-  size_t hwork_bytes;
+  float* linv;                    // inverse of the current diagonal block (128 x 128)
+  cudaStream_t side;              // the factorisation's diagonal blocks (high priority)
+  cudaEvent_t ev_fork, ev_join;
+  uint8_t *tcA, *tcB;             // prepared GEMM operands (tc_bytes each)
+  size_t tc_bytes;
   void* allocs[32];
   int nalloc;
   // column sweep scratch, grown on demand: W32 (n x k fp32), keep (n x k),
@@ -682,6 +923,7 @@ struct duo_calib {
   int z_ok;
   uint8_t* sw_keep;
   uint32_t *sw_keys, *sw_ctacnt;
+  uint8_t *sw_tcZ, *sw_tcEW;      // prepared operands of the lazy update
   int64_t sw_rows;
   uint32_t* sel_hist;             // SEL_DIGIT_BINS counters, zero between passes
   duo::calib::SelState* sel_state;
@@ -706,13 +948,10 @@ int map_cuda(cudaError_t e) {
   return DUO_ECUDA;
 }
 
-int map_blas(cublasStatus_t s) { return s == CUBLAS_STATUS_SUCCESS ? DUO_OK : DUO_ECUDA; }
-int map_solver(cusolverStatus_t s) { return s == CUSOLVER_STATUS_SUCCESS ? DUO_OK : DUO_ECUDA; }
-
 void release(duo_calib* h) {
-  if (h->blas) cublasDestroy(h->blas);
-  if (h->params) cusolverDnDestroyParams(h->params);
-  if (h->solver) cusolverDnDestroy(h->solver);
+  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+  if (h->ev_join) cudaEventDestroy(h->ev_join);
+  if (h->side) cudaStreamDestroy(h->side);
   for (int i = 0; i < h->nalloc; ++i) cudaFree(h->allocs[i]);
   cudaFree(h->sw_W32);
   cudaFree(h->sw_EW);
@@ -720,7 +959,8 @@ void release(duo_calib* h) {
   cudaFree(h->sw_keep);
   cudaFree(h->sw_keys);
   cudaFree(h->sw_ctacnt);
-  if (h->hwork) std::free(h->hwork);
+  cudaFree(h->sw_tcZ);
+  cudaFree(h->sw_tcEW);
   delete h;
 }
 
@@ -735,6 +975,98 @@ cudaError_t alloc(duo_calib* h, T** p, size_t count) {
 }
 
 bool aligned2(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 1u) == 0; }
+
+// Bytes of one prepared-operand buffer: H and G read k x m fp16 operands,
+// Q, D and the factorisation k x k (or k x 128, 128 x 128) fp32 ones, the
+// triangular inverse's doubling step s a batch of kp / (2 s) s x s blocks.
+size_t tc_scratch_bytes(int64_t k, int64_t m, int64_t kp) {
+  using duo::TC_F16;
+  using duo::TC_F32;
+  using duo::tc_operand_bytes;
+  size_t b = tc_operand_bytes(TC_F16, k, m, 1);
+  const size_t sizes[] = {tc_operand_bytes(TC_F32, k, k, 1), tc_operand_bytes(TC_F32, k, duo::calib::CHOL_NB, 1),
+                          tc_operand_bytes(TC_F32, duo::calib::CHOL_NB, duo::calib::CHOL_NB, 1)};
+  for (size_t v : sizes) b = v > b ? v : b;
+  for (int64_t sz = duo::calib::TRI_BASE; sz < kp; sz *= 2) {
+    const size_t v = tc_operand_bytes(TC_F32, sz, sz, kp / (2 * sz));
+    b = v > b ? v : b;
+  }
+  return b;
+}
+
+int map_tc(cudaError_t e) { return e == cudaSuccess ? DUO_OK : DUO_ECUDA; }
+
+// Blocked right-looking Cholesky factorisation of the leading k x k block of
+// the column-major factor buffer Hr (leading dimension kp), lower triangle,
+// in place; a failed pivot sets info[0].  Per 128-column block at j0, with
+// C11 and C11^-1 from chol_diag_kernel: the panel L21 = A21 C11^-T, then
+// the trailing update A22 -= L21 L21^T in two parts: first the next block
+// column, then (lower tiles) the rest.  The next block's diagonal kernel
+// only needs the first part, so it runs on the context's side stream (high
+// priority) while the rest of the update runs on `st`; `st` waits for it
+// before the next panel.  The GEMMs read prepared copies of their operands,
+// so the panel product may overwrite its own input.
+int factor_blocked(duo_calib* h, cudaStream_t st) {
+  using namespace duo::calib;
+  using duo::TC_F32;
+  const int k = (int)h->k, kp = (int)h->kp;
+  float* E = h->Hr;
+  cudaError_t e = cudaFuncSetAttribute(chol_diag_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, CHOL_SMEM);
+  if (e != cudaSuccess) return map_cuda(e);
+  chol_diag_kernel<<<1, CHOL_THREADS, CHOL_SMEM, st>>>(E, kp, 0, k < CHOL_NB ? k : CHOL_NB, h->linv, h->info);
+  e = cudaGetLastError();
+  // one prepared row tile of the 128-column panel: 2 chunks of 3 pieces
+  const size_t tile_bytes = duo::tc_operand_bytes(TC_F32, CHOL_NB, CHOL_NB, 1);
+  for (int j0 = 0; j0 + CHOL_NB < k && e == cudaSuccess; j0 += CHOL_NB) {
+    const int rest = k - j0 - CHOL_NB;                     // rows below the block
+    const int nb = rest < CHOL_NB ? rest : CHOL_NB;        // the next block's width
+    float* P = E + (j0 + CHOL_NB) + (size_t)j0 * kp;       // E(j0 + 128 + i, j0 + l)
+    duo::TcGemm g;
+    g.dtype = TC_F32;
+    g.M = rest;
+    g.N = g.K = CHOL_NB;
+    g.A = h->tcA;
+    g.B = h->tcB;
+    g.C = P;
+    g.c_m = 1;
+    g.c_n = kp;
+    e = duo::tc_prep(TC_F32, P, rest, CHOL_NB, 1, 1, kp, 0, h->tcA, st);
+    if (e == cudaSuccess) e = duo::tc_prep(TC_F32, h->linv, CHOL_NB, CHOL_NB, 1, CHOL_NB, 1, 0, h->tcB, st);
+    if (e == cudaSuccess) e = duo::launch_tc_gemm(g, st);   // L21(i, j) = sum_l A21(i, l) C11^-1(j, l)
+    if (e == cudaSuccess) e = duo::tc_prep(TC_F32, P, rest, CHOL_NB, 1, 1, kp, 0, h->tcA, st);
+    // the next block column: E(j0 + 128 + i, j0 + 128 + j) -= L21_i . L21_j, j < nb
+    duo::TcGemm t;
+    t.dtype = TC_F32;
+    t.M = rest;
+    t.N = nb;
+    t.K = CHOL_NB;
+    t.A = t.B = h->tcA;
+    t.C = E + (size_t)(j0 + CHOL_NB) * ((size_t)kp + 1);
+    t.c_m = 1;
+    t.c_n = kp;
+    t.alpha = -1.f;
+    t.beta = 1.f;
+    if (e == cudaSuccess) e = duo::launch_tc_gemm(t, st);
+    // the next diagonal block on the side stream
+    if (e == cudaSuccess) e = cudaEventRecord(h->ev_fork, st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_fork, 0);
+    if (e == cudaSuccess) {
+      chol_diag_kernel<<<1, CHOL_THREADS, CHOL_SMEM, h->side>>>(E, kp, j0 + CHOL_NB, nb, h->linv, h->info);
+      e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(h->ev_join, h->side);
+    // the rest of the trailing matrix (rows and columns from j0 + 256)
+    if (e == cudaSuccess && rest > CHOL_NB) {
+      t.M = t.N = rest - CHOL_NB;
+      t.A = t.B = h->tcA + tile_bytes;
+      t.C = E + (size_t)(j0 + 2 * CHOL_NB) * ((size_t)kp + 1);
+      t.lower = 1;
+      e = duo::launch_tc_gemm(t, st);
+    }
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, h->ev_join, 0);
+  }
+  return map_cuda(e);
+}
 
 }  // namespace
 
@@ -757,9 +1089,6 @@ int duo_calib_create(int64_t k, int64_t m, void* stream, duo_calib** out) {
     release(h);
     return code;
   };
-  if (cublasCreate(&h->blas) != CUBLAS_STATUS_SUCCESS) return fail(DUO_ECUDA);
-  if (cusolverDnCreate(&h->solver) != CUSOLVER_STATUS_SUCCESS) return fail(DUO_ECUDA);
-  if (cusolverDnCreateParams(&h->params) != CUSOLVER_STATUS_SUCCESS) return fail(DUO_ECUDA);
   const size_t kk = (size_t)k * k, km = (size_t)k * m;
   h->kp = duo::calib::tri_pad(k);
   cudaError_t e = cudaSuccess;
@@ -776,27 +1105,24 @@ int duo_calib_create(int64_t k, int64_t m, void* stream, duo_calib** out) {
   if (e == cudaSuccess) e = alloc(h, &h->key_hi, (size_t)k);
   if (e == cudaSuccess) e = alloc(h, &h->key_lo, (size_t)k);
   if (e == cudaSuccess) e = alloc(h, &h->perm, (size_t)k);
+  if (e == cudaSuccess) e = alloc(h, &h->rank, (size_t)k);
   if (e == cudaSuccess) e = alloc(h, &h->info, 2);
   if (e == cudaSuccess) e = alloc(h, &h->sel_hist, (size_t)duo::calib::SEL_DIGIT_BINS);
   if (e == cudaSuccess) e = alloc(h, &h->sel_state, 1);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->sel_hist, 0, sizeof(uint32_t) * duo::calib::SEL_DIGIT_BINS, st);
   if (e != cudaSuccess) return fail(map_cuda(e));
-  // cuSOLVER workspace of the factorisation.
-  size_t d1 = 0, h1 = 0;
-  cusolverDnSetStream(h->solver, st);
-  if (cusolverDnXpotrf_bufferSize(h->solver, h->params, CUBLAS_FILL_MODE_LOWER, k, CUDA_R_32F, h->Hr,
-                                  h->kp, CUDA_R_32F, &d1, &h1) != CUSOLVER_STATUS_SUCCESS)
-    return fail(DUO_ECUDA);
-  h->dwork_bytes = d1;
-  h->hwork_bytes = h1;
-  uint8_t* dw = nullptr;
-  e = alloc(h, &dw, h->dwork_bytes);
+  // the factorisation's side stream and its fork / join events
+  int prio_lo = 0, prio_hi = 0;
+  if (e == cudaSuccess) e = cudaDeviceGetStreamPriorityRange(&prio_lo, &prio_hi);
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->side, cudaStreamNonBlocking, prio_hi);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
+  // prepared GEMM operands: the largest of the precompute's products
+  h->tc_bytes = tc_scratch_bytes(k, m, h->kp);
+  if (e == cudaSuccess) e = alloc(h, &h->tcA, h->tc_bytes);
+  if (e == cudaSuccess) e = alloc(h, &h->tcB, h->tc_bytes);
+  if (e == cudaSuccess) e = alloc(h, &h->linv, (size_t)duo::calib::CHOL_NB * duo::calib::CHOL_NB);
   if (e != cudaSuccess) return fail(map_cuda(e));
-  h->dwork = dw;
-  if (h->hwork_bytes > 0) {
-    h->hwork = std::malloc(h->hwork_bytes);
-    if (h->hwork == nullptr) return fail(DUO_ENOMEM);
-  }
   e = cudaMemsetAsync(h->info, 0, 2 * sizeof(int), st);
   if (e == cudaSuccess) {
     const dim3 gp((unsigned)((h->kp + 255) / 256), (unsigned)h->kp);
@@ -832,33 +1158,51 @@ int duo_calib_precompute(duo_calib* h, const void* X_fp16_dev, int64_t keep, flo
   // 2. exact Hessian diagonal, a, act_order, dampening
   channel_stats_kernel<<<(k + 31) / 32, 32 * STAT_STRIDES, 0, st>>>(h->Xh, h->dX, k, m, h->key_hi,
                                                                     h->key_lo, h->a_orig);
-  rank_kernel<<<(k + RANK_THREADS - 1) / RANK_THREADS, RANK_THREADS, 0, st>>>(h->key_hi, h->key_lo, k,
-                                                                              act_order ? 1 : 0, h->perm);
+  e = cudaMemsetAsync(h->rank, 0, sizeof(int) * (size_t)k, st);
+  if (e != cudaSuccess) return map_cuda(e);
+  if (act_order)
+    rank_count_kernel<<<dim3((k + RANK_THREADS - 1) / RANK_THREADS, RANK_SPLIT), RANK_THREADS, 0, st>>>(
+        h->key_hi, h->key_lo, k, h->rank);
+  rank_place_kernel<<<(k + 255) / 256, 256, 0, st>>>(h->rank, k, act_order ? 1 : 0, h->perm);
   damp_kernel<<<1, 256, 0, st>>>(h->key_hi, h->key_lo, k, damp, h->dampadd);
   e = cudaGetLastError();
   if (e != cudaSuccess) return map_cuda(e);
-  // 3. H = X_hat X_hat^T and G = dX X_hat^T (fp16 in, fp32 accumulate):
-  //    the token-major buffers are column-major k x m matrices.
-  if (cublasSetStream(h->blas, st) != CUBLAS_STATUS_SUCCESS) return DUO_ECUDA;
-  const float one = 1.f, zero = 0.f;
-  int rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_N, CUBLAS_OP_T, k, k, m, &one, h->Xh, CUDA_R_16F, k,
-                                 h->Xh, CUDA_R_16F, k, &zero, h->H, CUDA_R_32F, k, CUBLAS_COMPUTE_32F,
-                                 CUBLAS_GEMM_DEFAULT));
+  // 3. H = X_hat X_hat^T and G = dX X_hat^T, fp16 operands: the
+  //    token-major buffers are column-major k x m matrices, so row i of an
+  //    operand is channel i (stride 1) over tokens (stride k).  Outputs
+  //    column-major: H[i + j k] = H_ij, and G transposed, G[i + j k] = G_ji
+  //    (the product X_hat dX^T).
+  using duo::TcGemm;
+  using duo::TC_F16;
+  using duo::TC_F32;
+  int rc = map_tc(duo::tc_prep(TC_F16, h->Xh, k, m, 1, 1, k, 0, h->tcA, st));
+  if (rc == DUO_OK) rc = map_tc(duo::tc_prep(TC_F16, h->dX, k, m, 1, 1, k, 0, h->tcB, st));
   if (rc != DUO_OK) return rc;
-  rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_N, CUBLAS_OP_T, k, k, m, &one, h->dX, CUDA_R_16F, k, h->Xh,
-                             CUDA_R_16F, k, &zero, h->G, CUDA_R_32F, k, CUBLAS_COMPUTE_32F,
-                             CUBLAS_GEMM_DEFAULT));
-  if (rc != DUO_OK) return rc;
+  {
+    TcGemm g;
+    g.dtype = TC_F16;
+    g.M = g.N = k;
+    g.K = m;
+    g.A = g.B = h->tcA;
+    g.C = h->H;
+    g.c_m = 1;
+    g.c_n = k;
+    rc = map_tc(duo::launch_tc_gemm(g, st));
+    if (rc != DUO_OK) return rc;
+    g.B = h->tcB;
+    g.C = h->G;
+    rc = map_tc(duo::launch_tc_gemm(g, st));
+    if (rc != DUO_OK) return rc;
+  }
   // 4. reorder and dampen, then L
   const dim3 g2((k + 255) / 256, k);
   const int kp = (int)h->kp;
   gather_kernel<<<g2, 256, 0, st>>>(h->H, h->G, h->perm, h->key_hi, h->key_lo, k, kp, h->dampadd, h->Hp,
                                     h->Hr, h->Gp);
-  e = cudaGetLastError();
+  e = cudaMemsetAsync(h->info, 0, 2 * sizeof(int), st);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return map_cuda(e);
-  if (cusolverDnSetStream(h->solver, st) != CUSOLVER_STATUS_SUCCESS) return DUO_ECUDA;
-  rc = map_solver(cusolverDnXpotrf(h->solver, h->params, CUBLAS_FILL_MODE_LOWER, k, CUDA_R_32F, h->Hr, kp,
-                                   CUDA_R_32F, h->dwork, h->dwork_bytes, h->hwork, h->hwork_bytes, h->info));
+  rc = factor_blocked(h, st);
   if (rc != DUO_OK) return rc;
   // C^-1 in place: base blocks, then one doubling step per level.  The
   // step's product B A^-1 goes to the H buffer (no longer needed; it holds
@@ -869,43 +1213,66 @@ int duo_calib_precompute(duo_calib* h, const void* X_fp16_dev, int64_t keep, flo
     tri_base_inverse_kernel<<<kp / TRI_BASE, TRI_BASE, 0, st>>>(h->Hr, kp);
     e = cudaGetLastError();
     if (e != cudaSuccess) return map_cuda(e);
-    const float minus_one = -1.f;
     for (int sz = TRI_BASE; sz < kp; sz *= 2) {
       const int batch = kp / (2 * sz);
-      const long long stride = 2LL * sz * ((long long)kp + 1);
-      float* A = h->Hr;
-      float* B = h->Hr + sz;
-      float* Dg = h->Hr + sz + (size_t)sz * kp;
-      rc = map_blas(cublasGemmStridedBatchedEx(h->blas, CUBLAS_OP_N, CUBLAS_OP_N, sz, sz, sz, &one, B,
-                                               CUDA_R_32F, kp, stride, A, CUDA_R_32F, kp, stride, &zero,
-                                               h->H, CUDA_R_32F, sz, (long long)sz * sz, batch, kL_COMPUTE,
-                                               CUBLAS_GEMM_DEFAULT));
-      if (rc != DUO_OK) return rc;
-      rc = map_blas(cublasGemmStridedBatchedEx(h->blas, CUBLAS_OP_N, CUBLAS_OP_N, sz, sz, sz, &minus_one,
-                                               Dg, CUDA_R_32F, kp, stride, h->H, CUDA_R_32F, sz,
-                                               (long long)sz * sz, &zero, B, CUDA_R_32F, kp, stride, batch,
-                                               kL_COMPUTE, CUBLAS_GEMM_DEFAULT));
+      const int64_t stride = 2LL * sz * ((int64_t)kp + 1);   // between diagonal block pairs
+      float* A = h->Hr;                                      // upper-left s x s block of a pair
+      float* B = h->Hr + sz;                                 // lower-left
+      float* Dg = h->Hr + sz + (size_t)sz * kp;              // lower-right
+      // T = B A^-1: T(i, j) = sum_l B(i, l) A^-1(l, j)
+      rc = map_tc(duo::tc_prep(TC_F32, B, sz, sz, batch, 1, kp, stride, h->tcA, st));
+      if (rc == DUO_OK) rc = map_tc(duo::tc_prep(TC_F32, A, sz, sz, batch, kp, 1, stride, h->tcB, st));
+      TcGemm g;
+      g.dtype = TC_F32;
+      g.M = g.N = g.K = sz;
+      g.batch = batch;
+      g.A = h->tcA;
+      g.B = h->tcB;
+      g.C = h->H;
+      g.c_m = 1;
+      g.c_n = sz;
+      g.c_bs = (int64_t)sz * sz;
+      if (rc == DUO_OK) rc = map_tc(duo::launch_tc_gemm(g, st));
+      // B <- -D^-1 T
+      if (rc == DUO_OK) rc = map_tc(duo::tc_prep(TC_F32, Dg, sz, sz, batch, 1, kp, stride, h->tcA, st));
+      if (rc == DUO_OK)
+        rc = map_tc(duo::tc_prep(TC_F32, h->H, sz, sz, batch, sz, 1, (int64_t)sz * sz, h->tcB, st));
+      g.C = B;
+      g.c_n = kp;
+      g.c_bs = stride;
+      g.alpha = -1.f;
+      if (rc == DUO_OK) rc = map_tc(duo::launch_tc_gemm(g, st));
       if (rc != DUO_OK) return rc;
     }
   }
   l_from_cinv_kernel<<<g2, 256, 0, st>>>(h->Hr, k, kp, h->L);
   e = cudaGetLastError();
   if (e != cudaSuccess) return map_cuda(e);
-  // 5. Q = Gp L.  Row-major buffers are the column-major transposes, so
-  //    Q^T = L^T Gp^T is a plain product of the two buffers.
-  rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_N, CUBLAS_OP_N, k, k, k, &one, h->L, CUDA_R_32F, k, h->Gp,
-                             CUDA_R_32F, k, &zero, h->Q, CUDA_R_32F, k, kL_COMPUTE,
-                             CUBLAS_GEMM_DEFAULT));
+  // 5. Q = Gp L (row-major buffers): Q^T(i, j) = sum_l L(l, i) Gp(j, l), so
+  //    with column-major output A(i, l) = L[l k + i] and B(j, l) = Gp[j k + l].
+  TcGemm g;
+  g.dtype = TC_F32;
+  g.M = g.N = g.K = k;
+  g.c_m = 1;
+  g.c_n = k;
+  g.A = h->tcA;
+  g.B = h->tcB;
+  rc = map_tc(duo::tc_prep(TC_F32, h->L, k, k, 1, 1, k, 0, h->tcA, st));
+  if (rc == DUO_OK) rc = map_tc(duo::tc_prep(TC_F32, h->Gp, k, k, 1, k, 1, 0, h->tcB, st));
+  g.C = h->Q;
+  if (rc == DUO_OK) rc = map_tc(duo::launch_tc_gemm(g, st));
   if (rc != DUO_OK) return rc;
   // 6. U, a (reordered), b, c and the score's column factor
   q_epilogue_kernel<<<k, EPI_THREADS, 0, st>>>(h->Q, h->L, h->a_orig, h->perm, k, h->U, h->a, h->b, h->c,
                                                h->col);
   e = cudaGetLastError();
   if (e != cudaSuccess) return map_cuda(e);
-  // 7. D = U L^T: D^T = L U^T, i.e. op(L buffer) = L and the U buffer as is.
-  rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_T, CUBLAS_OP_N, k, k, k, &one, h->L, CUDA_R_32F, k, h->U,
-                             CUDA_R_32F, k, &zero, h->D, CUDA_R_32F, k, kL_COMPUTE,
-                             CUBLAS_GEMM_DEFAULT));
+  // 7. D = U L^T (row-major): D^T(i, j) = sum_l L(i, l) U(j, l), A(i, l) =
+  //    L[i k + l], B(j, l) = U[j k + l].
+  rc = map_tc(duo::tc_prep(TC_F32, h->L, k, k, 1, k, 1, 0, h->tcA, st));
+  if (rc == DUO_OK) rc = map_tc(duo::tc_prep(TC_F32, h->U, k, k, 1, k, 1, 0, h->tcB, st));
+  g.C = h->D;
+  if (rc == DUO_OK) rc = map_tc(duo::launch_tc_gemm(g, st));
   return rc;
 }
 
@@ -916,6 +1283,9 @@ int duo_calib_status(const duo_calib* h, void* stream) {
   int info[2] = {0, 0};
   e = cudaMemcpy(info, h->info, sizeof(info), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return DUO_ECUDA;
+  unsigned int tc = 0;
+  if (duo::tc_gemm_take_status(&tc) != cudaSuccess) return DUO_ECUDA;
+  if (tc != 0) return DUO_ETIMEOUT;
   return info[0] != 0 ? DUO_ERANGE : DUO_OK;
 }
 
@@ -991,6 +1361,8 @@ int duo_calib_prune(duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw
     cudaFree(h->sw_keep);
     cudaFree(h->sw_keys);
     cudaFree(h->sw_ctacnt);
+    cudaFree(h->sw_tcEW);
+    h->sw_tcEW = nullptr;
     h->sw_W32 = nullptr;
     h->sw_EW = nullptr;
     h->sw_keep = nullptr;
@@ -1003,6 +1375,7 @@ int duo_calib_prune(duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw
     if (e == cudaSuccess) e = cudaMalloc(&h->sw_keys, (size_t)n * 128 * sizeof(uint32_t));
     if (e == cudaSuccess)
       e = cudaMalloc(&h->sw_ctacnt, ((size_t)n * 128 / SELM_PER_CTA + 1) * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMalloc(&h->sw_tcEW, duo::tc_operand_bytes(duo::TC_F32, n, 2 * 128, 1));
     if (e != cudaSuccess) return map_cuda(e);
     h->sw_rows = n;
   }
@@ -1010,6 +1383,8 @@ int duo_calib_prune(duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw
   float2* EW = h->sw_EW;
   if (h->sw_Z == nullptr) {
     e = cudaMalloc(&h->sw_Z, (size_t)k * k * sizeof(float2));
+    if (e == cudaSuccess && h->sw_tcZ == nullptr)
+      e = cudaMalloc(&h->sw_tcZ, duo::tc_operand_bytes(duo::TC_F32, k, 2 * 128, 1));
     if (e != cudaSuccess) return map_cuda(e);
     h->z_ok = 0;
   }
@@ -1023,8 +1398,6 @@ int duo_calib_prune(duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw
   load_permuted_kernel<<<gk, 256, 0, st>>>(static_cast<const uint16_t*>(W_fp16_dev), ldw, k, h->perm, W32);
   e = cudaFuncSetAttribute(block_sweep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SWEEP_SMEM);
   if (e != cudaSuccess) return map_cuda(e);
-  if (cublasSetStream(h->blas, st) != CUBLAS_STATUS_SUCCESS) return DUO_ECUDA;
-  const float one = 1.f;
   // rows (warps) per CTA of the in-block sweep: one CTA per SM, waves of 152
   const int64_t waves = (n + (int64_t)152 * SWEEP_ROWS - 1) / ((int64_t)152 * SWEEP_ROWS);
   const int rpc = (int)((n + 152 * waves - 1) / (152 * waves));
@@ -1051,14 +1424,27 @@ int duo_calib_prune(duo_calib* h, const void* W_fp16_dev, int64_t n, int64_t ldw
     const int nt = k - i - bj;   // trailing columns
     if (nt > 0) {
       // Lazy batch: W_T -= E L_T,blk^T - W_pre D_blk,T as one product of
-      // K = 2 B_j over the pairs: row-major buffers are column-major
-      // transposes, W_T^T (nt x n, ld k) += Z[T, blk]^T-view (nt x 2bj, read
-      // with OP_T from ld 2k) times {E, W_pre}^T (2bj x n, ld 2bj).
+      // K = 2 B_j over the pairs.  With column-major output over W32's rows
+      // (C(t, r) = W32[r k + i + bj + t]): A(t, l) = Z[i + bj + t] as floats
+      // (Z[q][j] = {-L_qj, D_jq}, pairs of block columns j), B(r, l) =
+      // {E, W_pre} of row r.
       const float* Zb = reinterpret_cast<const float*>(h->sw_Z) + (size_t)(i + bj) * 2 * k + 2 * (size_t)i;
-      int rc = map_blas(cublasGemmEx(h->blas, CUBLAS_OP_T, CUBLAS_OP_N, nt, (int)n, 2 * bj, &one, Zb,
-                                     CUDA_R_32F, 2 * k, EW, CUDA_R_32F, 2 * bj, &one, W32 + i + bj,
-                                     CUDA_R_32F, k, kL_COMPUTE, CUBLAS_GEMM_DEFAULT));
-      if (rc != DUO_OK) return rc;
+      duo::TcGemm g;
+      g.dtype = duo::TC_F32;
+      g.M = nt;
+      g.N = (int)n;
+      g.K = 2 * bj;
+      g.A = h->sw_tcZ;
+      g.B = h->sw_tcEW;
+      g.C = W32 + i + bj;
+      g.c_m = 1;
+      g.c_n = k;
+      g.beta = 1.f;
+      e = duo::tc_prep(duo::TC_F32, Zb, nt, 2 * bj, 1, 2 * (int64_t)k, 1, 0, h->sw_tcZ, st);
+      if (e == cudaSuccess)
+        e = duo::tc_prep(duo::TC_F32, EW, n, 2 * bj, 1, 2 * (int64_t)bj, 1, 0, h->sw_tcEW, st);
+      if (e == cudaSuccess) e = duo::launch_tc_gemm(g, st);
+      if (e != cudaSuccess) return map_cuda(e);
     }
   }
   store_unpermuted_kernel<<<gk, 256, 0, st>>>(W32, keepP, k, h->perm, Wout_dev, keep_dev);
