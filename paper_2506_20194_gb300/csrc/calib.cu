@@ -1061,6 +1061,7 @@ int factor_blocked(duo_calib* h, cudaStream_t st) {
       t.A = t.B = h->tcA + tile_bytes;
       t.C = E + (size_t)(j0 + 2 * CHOL_NB) * ((size_t)kp + 1);
       t.lower = 1;
+      t.max_ctas = -2;   // SMs left for the side stream's diagonal block
       e = duo::launch_tc_gemm(t, st);
     }
     if (e == cudaSuccess) e = cudaStreamWaitEvent(st, h->ev_join, 0);

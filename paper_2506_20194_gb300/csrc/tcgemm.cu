@@ -12,16 +12,17 @@
 // operand is then a single contiguous block of P x 16 KB that a bulk copy
 // (cp.async.bulk) moves into shared memory unchanged.
 //
-// tc_gemm_kernel: one CTA of 4 warps per 128 x 128 output tile, the fp32
-// accumulator in TMEM (128 columns).  Lane 0 of warp 0 streams the chunks of
-// A and B through an S-stage ring of shared-memory buffers (full / empty
+// tc_gemm_kernel: persistent, one CTA per SM (or fewer), 128 x 128 output
+// tiles handed out round-robin.  Lane 0 of warp 0 streams the chunks of A
+// and B through an S-stage ring of shared-memory buffers (full / empty
 // mbarriers, the copies completing transaction bytes on `full`); lane 0 of
 // warp 1 issues each chunk's MMAs (K = 16 each, 6 products per step for
-// fp32) and commits them to the stage's `empty` barrier, and after the last
-// chunk to `done`; then all four warps read TMEM with tcgen05.ld (warp w
-// holds rows 32 w .. 32 w + 31) and write C.  Every wait is bounded by a
-// wall-clock limit; a CTA that gives up still waits (bounded) for its copies
-// in flight and frees its TMEM.
+// fp32) into one of two TMEM accumulators and commits the stage to `empty`
+// and the finished tile to `acc_full`; warps 2..5 read the accumulator with
+// tcgen05.ld, write C and release it on `acc_empty`, so a tile's epilogue
+// runs under the next tile's MMAs.  Every wait is bounded by a wall-clock
+// limit; a CTA that gives up still waits (bounded) for its copies in flight
+// and frees its TMEM.
 #include <cstdint>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -33,7 +34,7 @@ namespace duo {
 namespace {
 
 constexpr int TG_M = 128, TG_N = 128, TG_K = 64;
-constexpr int TG_THREADS = 128;
+constexpr int TG_CTA_THREADS = 192;                // producer, MMA and four epilogue warps
 constexpr int TG_TILE = TG_M * TG_K * 2;            // bytes of one 128 x 64 16-bit tile
 constexpr int PREP_THREADS = 256;
 constexpr uint64_t TG_WAIT_NS = 1000000000ull;      // 1 s per bounded wait
@@ -182,35 +183,64 @@ __global__ void __launch_bounds__(PREP_THREADS) tc_prep_kernel(const T* __restri
   }
 }
 
+// Output tile t of the product (nt fastest, so that consecutive tiles share
+// their A rows): batch entry z, row tile mt, column tile nt; with `lower`
+// only tiles nt <= mt are enumerated.
+__device__ __forceinline__ void tile_of(int64_t t, int MT, int NT, int lower, int& z, int& mt, int& nt) {
+  if (!lower) {
+    const int64_t per = (int64_t)MT * NT, r = t % per;
+    z = (int)(t / per);
+    mt = (int)(r / NT);
+    nt = (int)(r % NT);
+  } else {
+    const int64_t per = (int64_t)MT * (MT + 1) / 2, r = t % per;
+    z = (int)(t / per);
+    int m = (int)((sqrtf(8.f * (float)r + 1.f) - 1.f) * 0.5f);
+    while ((int64_t)m * (m + 1) / 2 > r) --m;
+    while ((int64_t)(m + 1) * (m + 2) / 2 <= r) ++m;
+    mt = m;
+    nt = (int)(r - (int64_t)m * (m + 1) / 2);
+  }
+}
+
+// Persistent, warp-specialised: each CTA walks the tiles t = blockIdx.x,
+// blockIdx.x + gridDim.x, ...  Warp 0 (lane 0) streams every tile's chunks
+// through the S-stage ring; warp 1 (lane 0) issues the MMAs into one of two
+// TMEM accumulators (128 columns each) and commits the accumulator to
+// acc_full; warps 2..5 drain an accumulator (warp w reads TMEM lanes
+// 32 (w % 4) ..) into C and release it on acc_empty, so a tile's epilogue
+// overlaps the next tile's MMAs.
 template <int P>
-__global__ void __launch_bounds__(TG_THREADS, 1) tc_gemm_kernel(const TcGemm g) {
+__global__ void __launch_bounds__(TG_CTA_THREADS, 1) tc_gemm_kernel(const TcGemm g) {
   constexpr int NPROD = P == 1 ? 1 : 6;
   constexpr int S = P == 1 ? 4 : 2;                    // ring stages
   constexpr uint32_t OPB = P * TG_TILE;                // one operand's chunk
   constexpr uint32_t STB = 2 * OPB;                    // one stage: A chunk, then B chunk
   extern __shared__ __align__(1024) uint8_t sm[];
-  __shared__ __align__(8) uint64_t full[S], empty[S], done;
+  __shared__ __align__(8) uint64_t full[S], empty[S], acc_full[2], acc_empty[2], mma_done;
   __shared__ uint32_t tmem_base;
-  __shared__ int fail;
-  const int nt = blockIdx.x, mt = blockIdx.y, z = blockIdx.z;
-  if (g.lower && nt > mt) return;                      // tile entirely above the diagonal
+  __shared__ int fail_flag;
+  volatile int& fail = fail_flag;                      // set by any role that gives up
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nkc = (g.K + TG_K - 1) / TG_K;
-  const int64_t a_nrt = (g.M + TG_M - 1) / TG_M, b_nrt = (g.N + TG_N - 1) / TG_N;
-  const uint8_t* Ach = static_cast<const uint8_t*>(g.A) + ((int64_t)z * a_nrt + mt) * nkc * (int64_t)OPB;
-  const uint8_t* Bch = static_cast<const uint8_t*>(g.B) + ((int64_t)z * b_nrt + nt) * nkc * (int64_t)OPB;
+  const int MT = (g.M + TG_M - 1) / TG_M, NT = (g.N + TG_N - 1) / TG_N;
+  const int64_t ntiles = (int64_t)g.batch * (g.lower ? (int64_t)MT * (MT + 1) / 2 : (int64_t)MT * NT);
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       bar_init(&full[s], 1);
       bar_init(&empty[s], 1);
     }
-    bar_init(&done, 1);
+    for (int a = 0; a < 2; ++a) {
+      bar_init(&acc_full[a], 1);
+      bar_init(&acc_empty[a], 4);                      // one arrival per epilogue warp
+    }
+    bar_init(&mma_done, 1);
     fail = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 128;" ::"r"(su32(&tmem_base))
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(su32(&tmem_base))
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -221,90 +251,128 @@ __global__ void __launch_bounds__(TG_THREADS, 1) tc_gemm_kernel(const TcGemm g) 
 
   if (warp == 0) {
     if (lane == 0) {   // producer
-      int issued = 0;
-      for (int c = 0; c < nkc; ++c) {
-        const int s = c % S;
-        if (c >= S && !bar_wait(&empty[s], (uint32_t)(((c / S) - 1) & 1))) {
-          fail = 1;
-          break;
+      int64_t q = 0, issued = 0;                       // chunks over all of this CTA's tiles
+      for (int64_t t = blockIdx.x; t < ntiles && !fail; t += gridDim.x) {
+        int z, mt, nt;
+        tile_of(t, MT, NT, g.lower, z, mt, nt);
+        const uint8_t* Ach = static_cast<const uint8_t*>(g.A) + ((int64_t)z * MT + mt) * nkc * (int64_t)OPB;
+        const uint8_t* Bch = static_cast<const uint8_t*>(g.B) + ((int64_t)z * NT + nt) * nkc * (int64_t)OPB;
+        for (int c = 0; c < nkc; ++c, ++q) {
+          const int s = (int)(q % S);
+          const int64_t round = q / S;
+          if (round > 0 && !bar_wait(&empty[s], (uint32_t)((round - 1) & 1))) {
+            fail = 1;
+            break;
+          }
+          expect_tx(&full[s], STB);
+          bulk_copy(sm + s * STB, Ach + (int64_t)c * OPB, OPB, &full[s]);
+          bulk_copy(sm + s * STB + OPB, Bch + (int64_t)c * OPB, OPB, &full[s]);
+          issued = q + 1;
         }
-        expect_tx(&full[s], STB);
-        bulk_copy(sm + s * STB, Ach + (int64_t)c * OPB, OPB, &full[s]);
-        bulk_copy(sm + s * STB + OPB, Bch + (int64_t)c * OPB, OPB, &full[s]);
-        ++issued;
       }
       // every issued copy has landed before the CTA may exit
-      for (int c = issued > S ? issued - S : 0; c < issued; ++c)
+      for (int64_t c = issued > S ? issued - S : 0; c < issued; ++c)
         if (!bar_wait(&full[c % S], (uint32_t)((c / S) & 1))) fail = 1;
     }
     __syncwarp();
   } else if (warp == 1) {
     if (lane == 0) {   // MMA issuer
-      // (A piece, B piece) of each product, largest first
-      constexpr int PA[6] = {0, 0, 1, 0, 1, 2};
+      constexpr int PA[6] = {0, 0, 1, 0, 1, 2};         // (A piece, B piece) of each product
       constexpr int PB[6] = {0, 1, 0, 2, 1, 0};
       constexpr uint32_t ID = idesc_f16(P == 1 ? 0u : 1u);
-      for (int c = 0; c < nkc; ++c) {
-        const int s = c % S;
-        if (!bar_wait(&full[s], (uint32_t)((c / S) & 1))) {
+      int64_t q = 0, u = 0;
+      for (int64_t t = blockIdx.x; t < ntiles && !fail; t += gridDim.x, ++u) {
+        const int ab = (int)(u & 1);
+        const int64_t use = u >> 1;
+        if (use > 0 && !bar_wait(&acc_empty[ab], (uint32_t)((use - 1) & 1))) {
           fail = 1;
           break;
         }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t a0 = su32(sm + s * STB), b0 = a0 + OPB;
-#pragma unroll
-        for (int ks = 0; ks < TG_K / 16; ++ks) {
-#pragma unroll
-          for (int q = 0; q < NPROD; ++q) {
-            const uint32_t off = (uint32_t)ks * 256u;   // 16 columns = two core matrices along K
-            const uint32_t acc = (c > 0 || ks > 0 || q > 0) ? 1u : 0u;
-            mma(tmem, smem_desc(a0 + PA[q] * TG_TILE + off), smem_desc(b0 + PB[q] * TG_TILE + off), ID, acc);
+        const uint32_t d = tmem + (uint32_t)(ab * TG_N);
+        bool ok = true;
+        for (int c = 0; c < nkc; ++c, ++q) {
+          const int s = (int)(q % S);
+          if (!bar_wait(&full[s], (uint32_t)((q / S) & 1))) {
+            ok = false;
+            break;
           }
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          const uint32_t a0 = su32(sm + s * STB), b0 = a0 + OPB;
+#pragma unroll
+          for (int ks = 0; ks < TG_K / 16; ++ks) {
+#pragma unroll
+            for (int pr = 0; pr < NPROD; ++pr) {
+              const uint32_t off = (uint32_t)ks * 256u;   // 16 columns = two core matrices along K
+              const uint32_t acc = (c > 0 || ks > 0 || pr > 0) ? 1u : 0u;
+              mma(d, smem_desc(a0 + PA[pr] * TG_TILE + off), smem_desc(b0 + PB[pr] * TG_TILE + off), ID, acc);
+            }
+          }
+          commit(&empty[s]);
         }
-        commit(&empty[s]);
+        if (!ok) {
+          fail = 1;
+          break;
+        }
+        commit(&acc_full[ab]);   // arrives once this tile's MMAs have completed
       }
-      commit(&done);   // arrives once every MMA issued above has completed
+      // no MMA may still be writing TMEM when it is freed
+      commit(&mma_done);
+      if (!bar_wait(&mma_done, 0u)) fail = 1;
     }
     __syncwarp();
-  }
-  if (!bar_wait(&done, 0u)) fail = 1;
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-  __syncthreads();
-  if (!fail) {
-    const int r = mt * TG_M + 32 * warp + lane;
-    const int n0 = nt * TG_N;
-    float* C = g.C + (int64_t)z * g.c_bs;
-#pragma unroll 1
-    for (int c16 = 0; c16 < TG_N; c16 += 16) {
-      uint32_t v[16];
-      const uint32_t addr = tmem + ((uint32_t)(32 * warp) << 16) + (uint32_t)c16;
-      asm volatile(
-          "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, "
-          "[%16];"
-          : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-            "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]),
-            "=r"(v[15])
-          : "r"(addr));
-      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-      if (r < g.M) {
-        float* cr = C + (int64_t)r * g.c_m + (int64_t)(n0 + c16) * g.c_n;
-        float old[16];
-        // all 16 reads of C before any write: the stores may alias as far
-        // as the compiler knows, which would serialise each read behind the
-        // previous write
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          old[j] = (g.beta != 0.f && n0 + c16 + j < g.N) ? cr[(int64_t)j * g.c_n] : 0.f;
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (n0 + c16 + j < g.N) cr[(int64_t)j * g.c_n] = fmaf(g.beta, old[j], g.alpha * __uint_as_float(v[j]));
+  } else {   // epilogue: warps 2..5
+    const int quarter = warp & 3;                      // TMEM lanes 32 quarter .. 32 quarter + 31
+    int64_t u = 0;
+    for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x, ++u) {
+      const int ab = (int)(u & 1);
+      const bool got = bar_wait(&acc_full[ab], (uint32_t)((u >> 1) & 1));
+      if (!__all_sync(0xffffffffu, got) || fail) {
+        fail = 1;
+        break;
       }
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      int z, mt, nt;
+      tile_of(t, MT, NT, g.lower, z, mt, nt);
+      const int r = mt * TG_M + 32 * quarter + lane;
+      const int n0 = nt * TG_N;
+      float* C = g.C + (int64_t)z * g.c_bs;
+#pragma unroll 1
+      for (int c16 = 0; c16 < TG_N; c16 += 16) {
+        uint32_t v[16];
+        const uint32_t addr = tmem + (uint32_t)(ab * TG_N) + ((uint32_t)(32 * quarter) << 16) + (uint32_t)c16;
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, "
+            "[%16];"
+            : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+              "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]),
+              "=r"(v[15])
+            : "r"(addr));
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        if (r < g.M) {
+          float* cr = C + (int64_t)r * g.c_m + (int64_t)(n0 + c16) * g.c_n;
+          float old[16];
+          // all 16 reads of C before any write: the stores may alias as far
+          // as the compiler knows, which would serialise each read behind
+          // the previous write
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            old[j] = (g.beta != 0.f && n0 + c16 + j < g.N) ? cr[(int64_t)j * g.c_n] : 0.f;
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (n0 + c16 + j < g.N) cr[(int64_t)j * g.c_n] = fmaf(g.beta, old[j], g.alpha * __uint_as_float(v[j]));
+        }
+      }
+      // this warp's reads of the accumulator are done: release it
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(&acc_empty[ab])) : "memory");
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (warp == 0)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 128;" ::"r"(tmem) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tmem) : "memory");
 }
 
 int pieces(int dtype) { return dtype == TC_F16 ? 1 : 3; }
@@ -340,22 +408,30 @@ cudaError_t tc_prep(int dtype, const void* X, int64_t rows, int64_t K, int64_t b
 
 cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t st) {
   if (g.M <= 0 || g.N <= 0 || g.batch <= 0) return cudaSuccess;
-  if (g.K <= 0 || g.batch > 65535 || (g.M + TG_M - 1) / TG_M > 65535 || (g.N + TG_N - 1) / TG_N > 65535)
-    return cudaErrorInvalidValue;
+  if (g.K <= 0 || g.batch > 65535 || (g.lower && g.M != g.N)) return cudaErrorInvalidValue;
   if (g.A == nullptr || g.B == nullptr || g.C == nullptr || (reinterpret_cast<uintptr_t>(g.A) & 15u) != 0 ||
       (reinterpret_cast<uintptr_t>(g.B) & 15u) != 0)
     return cudaErrorInvalidValue;
-  const dim3 grid((unsigned)((g.N + TG_N - 1) / TG_N), (unsigned)((g.M + TG_M - 1) / TG_M), (unsigned)g.batch);
+  const int64_t MT = (g.M + TG_M - 1) / TG_M, NT = (g.N + TG_N - 1) / TG_N;
+  const int64_t ntiles = (int64_t)g.batch * (g.lower ? MT * (MT + 1) / 2 : MT * NT);
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  int64_t ctas = sms;
+  if (g.max_ctas > 0 && g.max_ctas < sms) ctas = g.max_ctas;
+  if (g.max_ctas < 0 && sms + g.max_ctas >= 1) ctas = sms + g.max_ctas;
+  if (ctas > ntiles) ctas = ntiles;
   if (g.dtype == TC_F16) {
     constexpr int smem = 4 * 2 * TG_TILE;
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(tc_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    tc_gemm_kernel<1><<<grid, TG_THREADS, smem, st>>>(g);
+    tc_gemm_kernel<1><<<(unsigned)ctas, TG_CTA_THREADS, smem, st>>>(g);
   } else if (g.dtype == TC_F32) {
     constexpr int smem = 2 * 2 * 3 * TG_TILE;
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(tc_gemm_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    tc_gemm_kernel<3><<<grid, TG_THREADS, smem, st>>>(g);
+    tc_gemm_kernel<3><<<(unsigned)ctas, TG_CTA_THREADS, smem, st>>>(g);
   } else {
     return cudaErrorInvalidValue;
   }

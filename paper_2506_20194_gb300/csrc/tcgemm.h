@@ -46,11 +46,13 @@ struct TcGemm {
   float* C = nullptr;
   int64_t c_m = 0, c_n = 0, c_bs = 0;
   float alpha = 1.f, beta = 0.f;
-  int lower = 0;
+  int lower = 0;      // lower tiles only (M == N)
+  int max_ctas = 0;   // persistent CTAs at most: 0 one per SM, n > 0 at most n, n < 0 all SMs but |n|
+                      // (SMs left free for kernels on other streams)
 };
 
-// Enqueues the product on `st`.  M, N or batch of 0 is a no-op; K < 1 or a
-// grid dimension above 65535 is cudaErrorInvalidValue.
+// Enqueues the product on `st`.  M, N or batch of 0 is a no-op; K < 1, a
+// batch above 65535 or `lower` with M != N is cudaErrorInvalidValue.
 cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t st);
 
 // Reads and clears the tensor-core GEMM status word: bit 0 is set when a
