@@ -447,3 +447,50 @@ cudaError_t tc_gemm_take_status(unsigned int* out) {
 }
 
 }  // namespace duo
+
+// ---------------------------------------------------------------------------
+// Internal, for the GEMM's own parity tests (not declared in the public
+// headers): prepares A and B (strided, fp16 when dtype == 0, fp32 when 1)
+// into temporary buffers, runs the product into C and synchronises.
+// Returns 0, -1 (invalid arguments), -4 (CUDA error) or -6 (a bounded wait
+// ran out), the codes of include/duo.h.
+// ---------------------------------------------------------------------------
+extern "C" int duo_test_tc_gemm(int dtype, int M, int N, int K, int batch, const void* A, int64_t a_m, int64_t a_k,
+                                int64_t a_bs, const void* B, int64_t b_n, int64_t b_k, int64_t b_bs, float* C,
+                                int64_t c_m, int64_t c_n, int64_t c_bs, float alpha, float beta, int lower,
+                                int max_ctas, void* stream) {
+  using namespace duo;
+  if ((dtype != TC_F16 && dtype != TC_F32) || M < 1 || N < 1 || K < 1 || batch < 1 || A == nullptr ||
+      B == nullptr || C == nullptr || (lower && M != N))
+    return -1;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  void *pa = nullptr, *pb = nullptr;
+  cudaError_t e = cudaMalloc(&pa, tc_operand_bytes(dtype, M, K, batch));
+  if (e == cudaSuccess) e = cudaMalloc(&pb, tc_operand_bytes(dtype, N, K, batch));
+  if (e == cudaSuccess) e = tc_prep(dtype, A, M, K, batch, a_m, a_k, a_bs, pa, st);
+  if (e == cudaSuccess) e = tc_prep(dtype, B, N, K, batch, b_n, b_k, b_bs, pb, st);
+  TcGemm g;
+  g.dtype = dtype;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.batch = batch;
+  g.A = pa;
+  g.B = pb;
+  g.C = C;
+  g.c_m = c_m;
+  g.c_n = c_n;
+  g.c_bs = c_bs;
+  g.alpha = alpha;
+  g.beta = beta;
+  g.lower = lower;
+  g.max_ctas = max_ctas;
+  if (e == cudaSuccess) e = launch_tc_gemm(g, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  cudaFree(pa);
+  cudaFree(pb);
+  if (e != cudaSuccess) return -4;
+  unsigned int v = 0;
+  if (tc_gemm_take_status(&v) != cudaSuccess) return -4;
+  return v != 0 ? -6 : 0;
+}

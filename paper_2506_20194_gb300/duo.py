@@ -72,6 +72,9 @@ def load_library(path: str | None = None):
     lib.duo_packed_status.argtypes = [vp, vp]
     # internal, for the failure-detection test (not part of include/duo.h)
     lib.duo_test_spmspv_blocked.argtypes = [vp, vp, i64, vp, ctypes.c_uint64, vp]
+    # internal, for the tensor-core GEMM's parity tests
+    lib.duo_test_tc_gemm.argtypes = [i32, i32, i32, i32, i32, vp, i64, i64, i64, vp, i64, i64, i64, vp, i64, i64,
+                                     i64, ctypes.c_float, ctypes.c_float, i32, i32, vp]
     lib.duo_copy.argtypes = [vp, vp, i64, vp]
     lib.duo_calib_create.argtypes = [i64, i64, vp, ctypes.POINTER(vp)]
     lib.duo_calib_precompute.argtypes = [vp, vp, i64, ctypes.c_float, i32, vp]
@@ -89,7 +92,7 @@ def load_library(path: str | None = None):
                  "duo_pack_cmb_noalloc", "duo_sparsify_threshold", "duo_spmspv_threshold",
                  "duo_calib_create", "duo_calib_precompute", "duo_calib_status", "duo_calib_export",
                  "duo_calib_score", "duo_calib_free", "duo_calib_prune", "duo_copy", "duo_calib_query",
-                 "duo_packed_status", "duo_test_spmspv_blocked"):
+                 "duo_packed_status", "duo_test_spmspv_blocked", "duo_test_tc_gemm"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
