@@ -11,6 +11,7 @@ namespace duo {
 
 constexpr int kMaxProblems = 4;
 constexpr int kMaxRuns = 128;   // (problem, segment) runs a launch may split by
+constexpr int kMaxCtaInfo = 256;   // CTAs whose run identity the launcher precomputes
 // Modes of the fused bitmask kernel.
 constexpr int CMB_LISTED = 0;   // kept list given by the caller
 constexpr int CMB_TOPK = 1;     // exact top-k selection in the kernel
@@ -26,6 +27,8 @@ struct CmbProb {
   int S;
   int G;                 // quantised formats: input-channel groups ceil(I / 128)
   float dens;            // non-zeros / (O * I): to estimate record sizes
+  uint32_t pf_bytes;     // set by the launcher: bytes of off[], 16-byte aligned (0: no warm-up)
+  uint32_t pf_chunk;     // set by the launcher: bytes of off[] each CTA warms in L2
 };
 
 struct CmbArgs {
@@ -53,6 +56,13 @@ struct CmbArgs {
                          // run has CTAs of its own: run r (items r*k .. r*k+k-1)
                          // goes to CTAs run_cta[r] .. run_cta[r+1]-1
   uint16_t run_cta[kMaxRuns + 1];
+  // set by the launcher when nruns > 0 and the grid has at most kMaxCtaInfo
+  // CTAs (else 0 and the kernel searches run_cta): per CTA its run r, the
+  // run's product p and segment s, the CTA's index m in the run and the
+  // run's CTA count n, packed as r | p << 8 | s << 10 | m << 32 | n << 48
+  // (one parameter load instead of a search)
+  int cta_info_ok;
+  uint64_t cta_info[kMaxCtaInfo];
 };
 
 struct Idx16Args {

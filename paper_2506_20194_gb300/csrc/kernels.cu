@@ -676,6 +676,18 @@ __device__ __forceinline__ Resolved resolve_item(const CmbArgs& a, const ItemCur
   return r;
 }
 
+// The run of this CTA: the r with run_cta[r] <= blockIdx.x < run_cta[r + 1]
+// (run_cta ascending from 0), by binary search over the kernel parameters.
+__device__ __forceinline__ int run_of_cta(const CmbArgs& a) {
+  int lo = 0, hi = a.nruns - 1;   // the answer lies in [lo, hi]
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if ((unsigned)a.run_cta[mid] <= blockIdx.x) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
 template <int MODE, int VB>
 __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArgs a) {
   constexpr bool FUSED = MODE != CMB_LISTED;   // the kernel builds its own kept list
@@ -715,12 +727,12 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   if (tid == 0) {
     abort_flag = 0;
     grid_open = 0;
-    for (int p = 0; p < a.np; ++p) {
-      const size_t bytes = align_up(((size_t)a.I * a.p[p].S + 1) * 4, 16);
-      const size_t lo = align_up(bytes * blockIdx.x / gridDim.x, 16);
-      const size_t hi = align_up(bytes * (blockIdx.x + 1) / gridDim.x, 16);
-      if (hi > lo) prefetch_l2(reinterpret_cast<const uint8_t*>(a.p[p].off) + lo, (uint32_t)(hi - lo));
-    }
+  }
+  if (warp == 0 && lane < a.np) {   // one lane per product, slices from the launcher
+    const CmbProb& P = a.p[lane];
+    const uint32_t lo = P.pf_chunk * blockIdx.x;
+    const uint32_t hi = lo + P.pf_chunk < P.pf_bytes ? lo + P.pf_chunk : P.pf_bytes;
+    if (hi > lo) prefetch_l2(reinterpret_cast<const uint8_t*>(P.off) + lo, hi - lo);
   }
   for (int i = tid; i < 2 * SEG_ROWS; i += CMB_THREADS) tile[i] = 0.f;
   if (MODE == CMB_TOPK) select_clear(sel);
@@ -731,13 +743,6 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     prefetch_line_l2(reinterpret_cast<const uint8_t*>(a.x) + 128 * tid);
   // Inputs, y and the grid barrier words may be the previous kernel's.
   griddep_wait();
-  // Generation of the grid barrier before this CTA arrives on it (read here,
-  // before any of this CTA's warps can arrive; issued ahead of the x loads
-  // so that the two round trips overlap).
-  unsigned int gen0 = 0;
-  if (tid == 0) {
-    gen0 = ld_relaxed_gpu(a.bar + 1);
-  }
   // Fused modes: x and the selection straight from registers when x fits
   // (select_window), else through shared memory.
   const bool regs = FUSED && select_window_ok<CMB_THREADS>(a.x, a.I);
@@ -750,18 +755,24 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     // Run r (product pr, segment sr): every CTA of it takes an equal share
     // of the run's kept channels in index order (select_window), or, on the
     // shared-memory path, the kept channels of its own channel range.
-    int r = 0;
-    while (r + 1 < a.nruns && (unsigned)a.run_cta[r + 1] <= blockIdx.x) ++r;
-    rn = a.run_cta[r + 1] - a.run_cta[r];
-    rm = blockIdx.x - a.run_cta[r];
+    if (a.cta_info_ok) {
+      const uint64_t ci = a.cta_info[blockIdx.x];
+      pr = (int)((ci >> 8) & 3u);
+      sr = (int)((ci >> 10) & 0x3FFFFFu);
+      rm = (uint32_t)((ci >> 32) & 0xFFFFu);
+      rn = (uint32_t)(ci >> 48);
+    } else {
+      const int r = run_of_cta(a);
+      rn = a.run_cta[r + 1] - a.run_cta[r];
+      rm = blockIdx.x - a.run_cta[r];
+      sr = r;
+      while (pr < a.np - 1 && sr >= a.p[pr].S) sr -= a.p[pr++].S;
+    }
     c0 = (int)((uint32_t)a.I * rm / rn);
     c1 = (int)((uint32_t)a.I * (rm + 1) / rn);
-    sr = r;
-    while (pr < a.np - 1 && sr >= a.p[pr].S) sr -= a.p[pr++].S;
     u0 = u1 = 0;
   } else if (a.nruns > 0) {
-    int r = 0;
-    while (r + 1 < a.nruns && (unsigned)a.run_cta[r + 1] <= blockIdx.x) ++r;
+    const int r = run_of_cta(a);
     const uint32_t n = a.run_cta[r + 1] - a.run_cta[r], m = blockIdx.x - a.run_cta[r];
     const uint32_t k = (uint32_t)a.k;   // k * m < 2^32: k <= 65535, m < 1024
     u0 = (uint32_t)r * k + k * m / n;
@@ -792,6 +803,12 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     u1 = (uint32_t)thresh_compact(xs, c0, c1, T, cut, klist, nullptr, sel->wcnt);
   }
   const int nv = (int)(u1 - u0);
+  // Generation of the grid barrier before this CTA arrives on it: read after
+  // the selection (no warp has arrived yet: consumers arrive after the role
+  // split) and used only once every copy is issued, so its round trip is
+  // off the path.
+  unsigned int gen0 = 0;
+  if (tid == 0) gen0 = ld_relaxed_gpu(a.bar + 1);
   // An item cursor at item u of this CTA.
   auto cursor_at = [&](uint32_t u) {
     ItemCursor c;
@@ -1268,6 +1285,15 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
       per_cta = std::max<int64_t>(per_cta, (a.k + n[q] - 1) / n[q]);
     }
     a.nruns = nruns;
+    a.cta_info_ok = grid <= kMaxCtaInfo ? 1 : 0;
+    if (a.cta_info_ok) {
+      int q = 0;
+      for (int p = 0; p < a.np; ++p)
+        for (int s = 0; s < a.p[p].S; ++s, ++q)
+          for (int m = 0; m < n[q]; ++m)
+            a.cta_info[a.run_cta[q] + m] = (uint64_t)q | (uint64_t)p << 8 | (uint64_t)s << 10 |
+                                           (uint64_t)m << 32 | (uint64_t)n[q] << 48;
+    }
     if (fused) {   // channel ranges: at most ceil(I / n) kept per CTA
       per_cta = 0;
       for (int q = 0; q < nruns; ++q) per_cta = std::max<int64_t>(per_cta, (a.I + n[q] - 1) / n[q]);
@@ -1307,6 +1333,13 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   DUO_CMB_PICK(CMB_LISTED, 4) DUO_CMB_PICK(CMB_TOPK, 4) DUO_CMB_PICK(CMB_THRESH, 4)
 #undef DUO_CMB_PICK
   if (kern == nullptr) return cudaErrorInvalidValue;
+  // L2 warm-up of the offset tables: each CTA one slice of every product's
+  for (int p = 0; p < a.np; ++p) {
+    const uint64_t bytes = align_up(((uint64_t)a.I * a.p[p].S + 1) * 4, 16);
+    const bool fits = bytes < (1ull << 31);
+    a.p[p].pf_bytes = fits ? (uint32_t)bytes : 0u;
+    a.p[p].pf_chunk = fits ? (uint32_t)align_up((bytes + grid - 1) / grid, 16) : 0u;
+  }
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
