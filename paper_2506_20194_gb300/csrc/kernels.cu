@@ -562,41 +562,59 @@ __device__ __forceinline__ void decode_record(const uint8_t* rec, uint16_t xb, f
 // Coded records (§5, weight-only quantisation): as decode_record / decode_two
 // with b-bit codes in place of the fp16 values; tab is the record's grid
 // table plus lane, so row 32 lane + t's grid is tab[32 t] (conflict-free).
+// The lane's codes come through a CodeWalk, (re)loaded every G positions
+// at the code index the mask prefix gives (independent loads).
 template <int VB>
 __device__ __forceinline__ void decode_record_q(const uint8_t* rec, uint16_t xb, const uint32_t* tab,
                                                 float (&acc)[32], int lane) {
+  constexpr int G = CodeWalk<VB>::G, NG = 32 / G;
   const uint32_t m = reinterpret_cast<const uint32_t*>(rec)[lane];
   const uint32_t c = __popc(m);
-  const uint32_t incl = warp_inclusive_scan(c, lane);
-  CodeWalk<VB> w;
-  w.init(rec + MASK_BYTES, incl - c);
+  const uint32_t c0 = warp_inclusive_scan(c, lane) - c;
+  CodeWalk<VB> w[NG];
 #pragma unroll
-  for (int t = 0; t < 32; ++t) {
-    const uint32_t bit = (m >> t) & 1u;
-    acc[t] = q_fma_sel(bit, w.at(), tab[32 * t], xb, acc[t]);
-    w.step(bit);
-  }
+  for (int g = 0; g < NG; ++g) w[g].load(rec + MASK_BYTES, c0 + (uint32_t)__popc(m & ((1ull << (G * g)) - 1u)));
+#pragma unroll
+  for (int g = 0; g < NG; ++g)
+#pragma unroll
+    for (int j = 0; j < G; ++j) {
+      const int t = G * g + j;
+      const uint32_t bit = (m >> t) & 1u;
+      acc[t] = q_fma_sel(bit, w[g].at(), tab[32 * t], xb, acc[t]);
+      w[g].step(bit);
+    }
 }
 
+// Two records of one group (one table) at once: one warp prefix sum serves
+// both masks (16-bit halves) and the two records' loads interleave.
 template <int VB>
-__device__ __forceinline__ void decode_two_q(const uint8_t* ra, uint16_t xa, const uint32_t* ta,
-                                             const uint8_t* rb, uint16_t xb, const uint32_t* tb,
-                                             float (&acc)[32], int lane) {
+__device__ __forceinline__ void decode_two_q(const uint8_t* ra, uint16_t xa, const uint8_t* rb, uint16_t xb,
+                                             const uint32_t* tab, float (&acc)[32], int lane) {
+  constexpr int G = CodeWalk<VB>::G, NG = 32 / G;
   const uint32_t ma = reinterpret_cast<const uint32_t*>(ra)[lane];
   const uint32_t mb = reinterpret_cast<const uint32_t*>(rb)[lane];
   const uint32_t c = (uint32_t)__popc(ma) | ((uint32_t)__popc(mb) << 16);
   const uint32_t ex = warp_inclusive_scan(c, lane) - c;
-  CodeWalk<VB> wa, wb;
-  wa.init(ra + MASK_BYTES, ex & 0xFFFFu);
-  wb.init(rb + MASK_BYTES, ex >> 16);
+  const uint32_t ca = ex & 0xFFFFu, cb = ex >> 16;
+  CodeWalk<VB> wa[NG], wb[NG];
 #pragma unroll
-  for (int t = 0; t < 32; ++t) {
-    const uint32_t ba = (ma >> t) & 1u, bb = (mb >> t) & 1u;
-    acc[t] = q_fma_sel(ba, wa.at(), ta[32 * t], xa, acc[t]);
-    acc[t] = q_fma_sel(bb, wb.at(), tb[32 * t], xb, acc[t]);
-    wa.step(ba);
-    wb.step(bb);
+  for (int g = 0; g < NG; ++g) {
+    const uint32_t below = (uint32_t)((1ull << (G * g)) - 1u);
+    wa[g].load(ra + MASK_BYTES, ca + (uint32_t)__popc(ma & below));
+    wb[g].load(rb + MASK_BYTES, cb + (uint32_t)__popc(mb & below));
   }
+#pragma unroll
+  for (int g = 0; g < NG; ++g)
+#pragma unroll
+    for (int j = 0; j < G; ++j) {
+      const int t = G * g + j;
+      const uint32_t ba = (ma >> t) & 1u, bb = (mb >> t) & 1u;
+      const uint32_t e = tab[32 * t];
+      acc[t] = q_fma_sel(ba, wa[g].at(), e, xa, acc[t]);
+      acc[t] = q_fma_sel(bb, wb[g].at(), e, xb, acc[t]);
+      wa[g].step(ba);
+      wb[g].step(bb);
+    }
 }
 
 // Item cursor: (product p, segment s, kept rank i) of a linear item index.
@@ -1046,6 +1064,8 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     // Coded formats: the grid table of an item's group (its table number is
     // in the slot's xval word), waited for once per table; and the count of
     // released items, which tells the producer when a table buffer is free.
+    // (Copying the group's grid into 32 registers per lane measured no faster
+    // than reading it from shared memory per row.)
     int ncons = 0, cur_seq = -1;
     const uint32_t* tcur = nullptr;
     auto table_for = [&](uint32_t seq) -> const uint32_t* {
@@ -1115,7 +1135,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
               const uint32_t xa = xval[sc.slot], xb2 = xval[sc2.slot];
               const uint32_t* tb = table_for(xa >> 16);
               if (tb != nullptr) {
-                decode_two_q<VB>(ring + (size_t)sc.slot * slot_bytes, (uint16_t)xa, tb,
+                decode_two_q<VB>(ring + (size_t)sc.slot * slot_bytes, (uint16_t)xa,
                                  ring + (size_t)sc2.slot * slot_bytes, (uint16_t)xb2, tb, acc, lane);
                 any = true;
               }
