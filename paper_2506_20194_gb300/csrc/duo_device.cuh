@@ -757,18 +757,17 @@ __device__ __noinline__ int select_window(const uint16_t* x, int I, int k, int t
 #pragma unroll
   for (int c = 0; c < 4; ++c) {
     if (c < NCH) {
-      uint32_t g0 = gbase + field(ex[c >> 1], c), e0 = ebase + field(ex[2 + (c >> 1)], c);
-      uint32_t bits = gb[c] | eb[c];
-      while (bits) {   // the chunk's channels with key >= T, in order
-        const int h = __ffs(bits) - 1;
+      // the chunk's 8 channels, each ranked on its own (no loop-carried
+      // find-first-set): kept when key > T, or key == T within the first q
+      const uint32_t g0 = gbase + field(ex[c >> 1], c), e0 = ebase + field(ex[2 + (c >> 1)], c);
+      const uint32_t gbc = gb[c], ebc = eb[c];
+#pragma unroll
+      for (int h = 0; h < 8; ++h) {
         const uint32_t below = (1u << h) - 1u;
-        const uint32_t g = g0 + (uint32_t)__popc(gb[c] & below), e = e0 + (uint32_t)__popc(eb[c] & below);
-        const bool isg = (gb[c] >> h) & 1u;
-        if (isg || e < qq) {
-          const uint32_t r = g + (e < qq ? e : qq);
-          if (r >= R0 && r < R1) klist[r - R0] = (uint16_t)(8 * (tid + c * ST_THREADS) + h);
-        }
-        bits &= bits - 1;
+        const uint32_t g = g0 + (uint32_t)__popc(gbc & below), e = e0 + (uint32_t)__popc(ebc & below);
+        const bool kept = ((gbc >> h) & 1u) || (((ebc >> h) & 1u) && e < qq);
+        const uint32_t r = g + (e < qq ? e : qq);
+        if (kept && r >= R0 && r < R1) klist[r - R0] = (uint16_t)(8 * (tid + c * ST_THREADS) + h);
       }
     }
     gbase += field(tot[c >> 1], c);

@@ -759,6 +759,10 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   // is what the loads after the wait see.
   if (FUSED && tid < (2 * a.I + 127) / 128)
     prefetch_line_l2(reinterpret_cast<const uint8_t*>(a.x) + 128 * tid);
+  // This CTA's run identity (a kernel parameter, not the previous kernel's
+  // output): read before the wait so that its cold parameter-cache miss
+  // overlaps the wait.
+  const uint64_t cinfo = (FUSED && a.cta_info_ok) ? a.cta_info[blockIdx.x] : 0ull;
   // Inputs, y and the grid barrier words may be the previous kernel's.
   griddep_wait();
   // Fused modes: x and the selection straight from registers when x fits
@@ -774,7 +778,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     // of the run's kept channels in index order (select_window), or, on the
     // shared-memory path, the kept channels of its own channel range.
     if (a.cta_info_ok) {
-      const uint64_t ci = a.cta_info[blockIdx.x];
+      const uint64_t ci = cinfo;
       pr = (int)((ci >> 8) & 3u);
       sr = (int)((ci >> 10) & 0x3FFFFFu);
       rm = (uint32_t)((ci >> 32) & 0xFFFFu);
