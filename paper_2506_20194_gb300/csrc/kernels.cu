@@ -694,6 +694,15 @@ __device__ __forceinline__ Resolved resolve_item(const CmbArgs& a, const ItemCur
   return r;
 }
 
+// Whether consumers may decode two records at once (one scan for both
+// masks, interleaved loads) when the ring allows it.  Measured on the 7B
+// layer (us per layer, with / without): fp16 64.5 / 66.4, 8-bit codes
+// 85.4 / 86.7, 4-bit codes 103.3 / 101.4 -- so 4-bit launches decode one
+// record at a time (and their kernels carry no pair code).
+#ifndef CMB_PAIRS
+#define CMB_PAIRS 1
+#endif
+
 // The run of this CTA: the r with run_cta[r] <= blockIdx.x < run_cta[r + 1]
 // (run_cta ascending from 0), by binary search over the kernel parameters.
 __device__ __forceinline__ int run_of_cta(const CmbArgs& a) {
@@ -1118,7 +1127,7 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
       // this consumer's items in pairs, then alone
       SlotCursor sc, sc2;
       sc.set(v, nslot);
-      if (a.group >= 2) {
+      if (CMB_PAIRS && VB != 4 && a.group >= 2) {
         sc2.set(v + CMB_NC, nslot);
         for (; v + CMB_NC < vb; v += 2 * CMB_NC) {   // pairs
           if constexpr (!QUANT) {
@@ -1344,7 +1353,7 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   // Pairs (waiting for more records costs more than it gains); coded
   // formats pair only items of one group, which a consumer can tell ahead
   // only from the kept list in shared memory (fused modes).
-  a.group = (nslot >= 2 * CMB_NC && (fused || !quant)) ? 2 : 1;
+  a.group = (CMB_PAIRS && a.vbits != 4 && nslot >= 2 * CMB_NC && (fused || !quant)) ? 2 : 1;
   a.nslot = nslot;
   a.slot_bytes = slot_bytes;
   const size_t smem = cmb_layout(a.I, fused, a.list_cap, nslot, slot_bytes, quant).total;
