@@ -38,8 +38,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch of
 # the fused kernel from one ncu capture, valid only for the kernel source it
 # was taken on (sha256 of kernels.cu + duo_device.cuh, first 16 hex digits).
-TRAFFIC = {"sha": "5dd7468aa091b8d7",
-           "per_launch_bytes": [29114624.0, 9761280.0, 51836672.0, 26118656.0]}
+TRAFFIC = {"sha": "070f7884de7c29b3",
+           "per_launch_bytes": [29117696.0, 9760000.0, 51918848.0, 26117632.0]}
 
 
 def parse():

@@ -590,14 +590,15 @@ __device__ __forceinline__ bool select_window_ok(const uint16_t* x, int I) {
 //    fewer than q equal keys before it) has rank #(key > T before it) +
 //    min(q, #(key == T before it)); each thread writes its kept channels
 //    whose rank lies in this CTA's window [K m / nr, K (m + 1) / nr), K the
-//    number kept, to klist (ascending).  Every CTA of a run thus gets the
-//    same number of channels (+-1) however x is spread.
+//    number kept (m = bits 32..47 of `run`, this CTA's index in its run,
+//    nr = bits 48..63, the run's CTAs), to klist (ascending).  Every CTA of
+//    a run thus gets the same number of channels (+-1) however x is spread.
 // Returns the window size; ends with a barrier.  NCH = ceil((I / 8) /
 // NT), 1..4 (select_window_ok() tells whether it fits).  All NT threads of the
 // block take part; tmp needs 6 NT / 32 words.
 template <bool TOPK, int NCH, int NT>
 __device__ __noinline__ int select_window(const uint16_t* x, int I, int k, int tau_key,
-                                             uint16_t* xs, SelShared* sh, uint32_t m, uint32_t nr,
+                                             uint16_t* xs, SelShared* sh, uint64_t run,
                                              uint16_t* klist, uint32_t* tmp) {
   constexpr int ST_THREADS = NT, ST_WARPS = NT / 32;
   static_assert(ST_WARPS * 128 == SEL_BINS, "each warp sums 128 histogram bins");
@@ -680,15 +681,25 @@ __device__ __noinline__ int select_window(const uint16_t* x, int I, int k, int t
       }
       const int C = 128 * W + 4 * L + __shfl_sync(FULL_MASK, b, L);
       const uint32_t aboveC = __shfl_sync(FULL_MASK, above, L);
-      // the keys of bin C, by their low 4 bits
+      // the keys of bin C, by their low 4 bits.  A chunk is tested two keys
+      // a word first: a 16-bit half of (key >> 4) ^ C is 0 exactly for a key
+      // of bin C, and subtracting 1 then sets the half's top bit (the halves
+      // hold 11 bits; a borrow from the low half can also set the high
+      // half's: a false alarm, which the exact loop rules out)
+      const uint32_t CC = (uint32_t)C * 0x10001u;
 #pragma unroll
       for (int c = 0; c < NCH; ++c)
-        if (have[c])
+        if (have[c]) {
+          uint32_t z = 0;
 #pragma unroll
-          for (int h = 0; h < 8; ++h) {
-            const int key = key_at(c, h);
-            if ((key >> 4) == C) atomicAdd(&sh->sub[key & 15], 1u);
-          }
+          for (int u = 0; u < 4; ++u) z |= (((w[4 * c + u] >> 4) & 0x07FF07FFu) ^ CC) - 0x00010001u;
+          if (z & 0x80008000u)
+#pragma unroll
+            for (int h = 0; h < 8; ++h) {
+              const int key = key_at(c, h);
+              if ((key >> 4) == C) atomicAdd(&sh->sub[key & 15], 1u);
+            }
+        }
       if (tail && (int)((xt & 0x7FFFu) >> 4) == C) atomicAdd(&sh->sub[xt & 15u], 1u);
       __syncthreads();
       // T and q, in every warp: the 16 keys of bin C from the top
@@ -705,19 +716,28 @@ __device__ __noinline__ int select_window(const uint16_t* x, int I, int k, int t
       q = (int)(need - __shfl_sync(FULL_MASK, sfx - sv, bb));   // >= 1
     }
   }
-  // per chunk: bits and counts of key > T and key == T
+  // per chunk: bits and counts of key > T and key == T, two keys a word:
+  // with the sign bit set, (key | 0x8000) - t has bit 15 set exactly when
+  // key >= t (0 <= t <= 0x8000: no borrow leaves the half), so t = T + 1
+  // gives key > T and t = max(T, 0) key >= T; the words' bits 15 and 31 are
+  // then gathered into the chunk's 8-bit masks (bit h: channel h)
   uint32_t gb[NCH], eb[NCH];
   uint32_t p[5] = {0u, 0u, 0u, 0u, 0u};   // gt of chunks 0|1, 2|3, eq 0|1, 2|3, {gt, eq} of the tail
+  const uint32_t T1 = (uint32_t)(T + 1) * 0x10001u, T0 = (uint32_t)(T < 0 ? 0 : T) * 0x10001u;
 #pragma unroll
   for (int c = 0; c < NCH; ++c) {
     uint32_t g = 0, e = 0;
-    if (have[c])
+    if (have[c]) {
 #pragma unroll
-      for (int h = 0; h < 8; ++h) {
-        const int key = key_at(c, h);
-        g |= (key > T ? 1u : 0u) << h;
-        e |= (key == T ? 1u : 0u) << h;
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t o = w[4 * c + u] | 0x80008000u;
+        const uint32_t gw = (o - T1) & 0x80008000u, ew = (o - T0) & ~gw & 0x80008000u;
+        g |= gw >> (15 - 2 * u);
+        e |= ew >> (15 - 2 * u);
       }
+      g = (g | (g >> 15)) & 0xFFu;
+      e = (e | (e >> 15)) & 0xFFu;
+    }
     gb[c] = g;
     eb[c] = e;
     p[c >> 1] |= (uint32_t)__popc(g) << (16 * (c & 1));
@@ -726,22 +746,30 @@ __device__ __noinline__ int select_window(const uint16_t* x, int I, int k, int t
   const int tkey = (int)(xt & 0x7FFFu);
   const uint32_t tg = (tail && tkey > T) ? 1u : 0u, te = (tail && tkey == T) ? 1u : 0u;
   p[4] = tg | (te << 16);
-  // block exclusive scan of the five packed counters (16-bit fields: at
-  // most 8 ST_THREADS per field); every warp scans the warp totals itself
+  // block exclusive scan of the packed counters (16-bit fields: at most
+  // 8 ST_THREADS per field).  Words 1 and 3 (chunks 2 and 3) exist only for
+  // NCH > 2 and word 4 only when I % 8 != 0 (block-uniform); the others are
+  // zero and not scanned.  Across warps: the exclusive prefix and the total
+  // of the warp totals, each one warp reduction.
+  const bool ftail = (I & 7) != 0;
+  auto live = [&](int f) { return (f & 1) == 0 ? (f < 4 || ftail) : NCH > 2; };
   uint32_t incl[5];
 #pragma unroll
-  for (int f = 0; f < 5; ++f) incl[f] = warp_inclusive_scan(p[f], lane);
+  for (int f = 0; f < 5; ++f) incl[f] = live(f) ? warp_inclusive_scan(p[f], lane) : 0u;
   if (lane == 31)
 #pragma unroll
-    for (int f = 0; f < 5; ++f) tmp[ST_WARPS + 5 * wid + f] = incl[f];
+    for (int f = 0; f < 5; ++f)
+      if (live(f)) tmp[ST_WARPS + 5 * wid + f] = incl[f];
   __syncthreads();
   uint32_t ex[5], tot[5];
 #pragma unroll
   for (int f = 0; f < 5; ++f) {
-    const uint32_t v = lane < ST_WARPS ? tmp[ST_WARPS + 5 * lane + f] : 0u;
-    const uint32_t in = warp_inclusive_scan(v, lane);
-    ex[f] = __shfl_sync(FULL_MASK, in - v, wid) + incl[f] - p[f];
-    tot[f] = __shfl_sync(FULL_MASK, in, ST_WARPS - 1);
+    ex[f] = tot[f] = 0u;
+    if (live(f)) {
+      const uint32_t v = lane < ST_WARPS ? tmp[ST_WARPS + 5 * lane + f] : 0u;
+      ex[f] = __reduce_add_sync(FULL_MASK, lane < wid ? v : 0u) + incl[f] - p[f];
+      tot[f] = __reduce_add_sync(FULL_MASK, v);
+    }
   }
   auto field = [](uint32_t v, int c) { return (v >> (16 * (c & 1))) & 0xFFFFu; };
   uint32_t GT = (tot[4] & 0xFFFFu), EQ = (tot[4] >> 16);
@@ -752,6 +780,7 @@ __device__ __noinline__ int select_window(const uint16_t* x, int I, int k, int t
   }
   const uint32_t qq = (uint32_t)q;
   const uint32_t K = GT + (EQ < qq ? EQ : qq);
+  const uint32_t m = (uint32_t)(run >> 32) & 0xFFFFu, nr = (uint32_t)(run >> 48);
   const uint32_t R0 = K * m / nr, R1 = K * (m + 1) / nr;
   uint32_t gbase = 0, ebase = 0;
 #pragma unroll
@@ -761,13 +790,19 @@ __device__ __noinline__ int select_window(const uint16_t* x, int I, int k, int t
       // find-first-set): kept when key > T, or key == T within the first q
       const uint32_t g0 = gbase + field(ex[c >> 1], c), e0 = ebase + field(ex[2 + (c >> 1)], c);
       const uint32_t gbc = gb[c], ebc = eb[c];
+      // the chunk's kept channels take ranks from r0c on, at most 8 of them:
+      // only chunks that can reach this CTA's window [R0, R1) are ranked
+      // (a few threads of the CTA; the others skip it)
+      const uint32_t r0c = g0 + (e0 < qq ? e0 : qq);
+      if (r0c < R1 && r0c + 8u > R0) {
 #pragma unroll
-      for (int h = 0; h < 8; ++h) {
-        const uint32_t below = (1u << h) - 1u;
-        const uint32_t g = g0 + (uint32_t)__popc(gbc & below), e = e0 + (uint32_t)__popc(ebc & below);
-        const bool kept = ((gbc >> h) & 1u) || (((ebc >> h) & 1u) && e < qq);
-        const uint32_t r = g + (e < qq ? e : qq);
-        if (kept && r >= R0 && r < R1) klist[r - R0] = (uint16_t)(8 * (tid + c * ST_THREADS) + h);
+        for (int h = 0; h < 8; ++h) {
+          const uint32_t below = (1u << h) - 1u;
+          const uint32_t g = g0 + (uint32_t)__popc(gbc & below), e = e0 + (uint32_t)__popc(ebc & below);
+          const bool kept = ((gbc >> h) & 1u) || (((ebc >> h) & 1u) && e < qq);
+          const uint32_t r = g + (e < qq ? e : qq);
+          if (kept && r >= R0 && r < R1) klist[r - R0] = (uint16_t)(8 * (tid + c * ST_THREADS) + h);
+        }
       }
     }
     gbase += field(tot[c >> 1], c);

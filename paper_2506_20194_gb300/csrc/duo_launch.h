@@ -36,6 +36,8 @@ struct CmbArgs {
   int np;
   int I;
   int k;
+  int cta_info_ok;       // set by the launcher: cta_info holds every CTA's run (see below);
+                         // next to I and x, whose parameter line the kernel reads first
   const uint16_t* x;     // fused mode: fp16 bits [I]
   const uint16_t* kidx;  // listed mode: uint16 [k]
   const uint16_t* kval;  // listed mode: fp16 bits [k]
@@ -57,11 +59,10 @@ struct CmbArgs {
                          // goes to CTAs run_cta[r] .. run_cta[r+1]-1
   uint16_t run_cta[kMaxRuns + 1];
   // set by the launcher when nruns > 0 and the grid has at most kMaxCtaInfo
-  // CTAs (else 0 and the kernel searches run_cta): per CTA its run r, the
-  // run's product p and segment s, the CTA's index m in the run and the
-  // run's CTA count n, packed as r | p << 8 | s << 10 | m << 32 | n << 48
-  // (one parameter load instead of a search)
-  int cta_info_ok;
+  // CTAs (cta_info_ok = 1; else 0 and the kernel searches run_cta): per CTA
+  // its run r, the run's product p and segment s, the CTA's index m in the
+  // run and the run's CTA count n, packed as r | p << 8 | s << 10 | m << 32 |
+  // n << 48 (one parameter load instead of a search)
   uint64_t cta_info[kMaxCtaInfo];
 };
 

@@ -755,13 +755,15 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     abort_flag = 0;
     grid_open = 0;
   }
-  if (warp == 0 && lane < a.np) {   // one lane per product, slices from the launcher
-    const CmbProb& P = a.p[lane];
+  if (warp < a.np && lane == 0) {   // one warp per product (its parameters: one
+                                    // uniform load each), slices from the launcher
+    const CmbProb& P = a.p[warp];
     const uint32_t lo = P.pf_chunk * blockIdx.x;
     const uint32_t hi = lo + P.pf_chunk < P.pf_bytes ? lo + P.pf_chunk : P.pf_bytes;
     if (hi > lo) prefetch_l2(reinterpret_cast<const uint8_t*>(P.off) + lo, hi - lo);
   }
-  for (int i = tid; i < 2 * SEG_ROWS; i += CMB_THREADS) tile[i] = 0.f;
+  for (int i = tid; i < SEG_ROWS / 2; i += CMB_THREADS)   // 2 SEG_ROWS floats, 16 B a store
+    reinterpret_cast<float4*>(tile)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
   if (MODE == CMB_TOPK) select_clear(sel);
   // x into L2 while the previous kernel finishes: a prefetch reads nothing
   // into this CTA, and L2 is coherent, so a later write to x by that kernel
@@ -780,27 +782,22 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   if (FUSED && !regs) load_x_to_smem(xs, a.x, a.I);
   uint32_t u0, u1;   // this CTA's items (32-bit: the launcher keeps counts < 2^31)
   int r0 = 0;        // kept rank of its first item
-  int pr = 0, sr = 0, c0 = 0, c1 = 0;   // fused modes: run (product, segment), channel range
-  uint32_t rm = 0, rn = 1;               // fused modes: this CTA's index in its run, the run's CTAs
+  int pr = 0, sr = 0;   // fused modes: run (product, segment)
+  // Fused modes: the run identity p << 8 | s << 10 | m << 32 | n << 48 (this
+  // CTA is the m-th of the n CTAs of product p's segment s).  Every CTA of a
+  // run takes an equal share of the run's kept channels in index order
+  // (select_window), or, on the shared-memory path, the kept channels of its
+  // own channel range.  The launcher's word is decoded only where it is
+  // used, so that its parameter load overlaps the loads of x.
+  uint64_t ci = cinfo;
   if (FUSED) {
-    // Run r (product pr, segment sr): every CTA of it takes an equal share
-    // of the run's kept channels in index order (select_window), or, on the
-    // shared-memory path, the kept channels of its own channel range.
-    if (a.cta_info_ok) {
-      const uint64_t ci = cinfo;
-      pr = (int)((ci >> 8) & 3u);
-      sr = (int)((ci >> 10) & 0x3FFFFFu);
-      rm = (uint32_t)((ci >> 32) & 0xFFFFu);
-      rn = (uint32_t)(ci >> 48);
-    } else {
+    if (!a.cta_info_ok) {
       const int r = run_of_cta(a);
-      rn = a.run_cta[r + 1] - a.run_cta[r];
-      rm = blockIdx.x - a.run_cta[r];
-      sr = r;
-      while (pr < a.np - 1 && sr >= a.p[pr].S) sr -= a.p[pr++].S;
+      int p = 0, sg = r;
+      while (p < a.np - 1 && sg >= a.p[p].S) sg -= a.p[p++].S;
+      ci = (uint64_t)p << 8 | (uint64_t)sg << 10 | (uint64_t)(blockIdx.x - a.run_cta[r]) << 32 |
+           (uint64_t)(a.run_cta[r + 1] - a.run_cta[r]) << 48;
     }
-    c0 = (int)((uint32_t)a.I * rm / rn);
-    c1 = (int)((uint32_t)a.I * (rm + 1) / rn);
     u0 = u1 = 0;
   } else if (a.nruns > 0) {
     const int r = run_of_cta(a);
@@ -821,17 +818,23 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
     const int nch = ((a.I >> 3) + CMB_THREADS - 1) / CMB_THREADS;
     const int tk = (int)a.tau_key;
     int nw;
-    if (nch <= 1) nw = select_window<TK, 1, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, rm, rn, klist, sel->tmp);
-    else if (nch == 2) nw = select_window<TK, 2, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, rm, rn, klist, sel->tmp);
-    else if (nch == 3) nw = select_window<TK, 3, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, rm, rn, klist, sel->tmp);
-    else nw = select_window<TK, 4, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, rm, rn, klist, sel->tmp);
+    if (nch <= 1) nw = select_window<TK, 1, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, ci, klist, sel->tmp);
+    else if (nch == 2) nw = select_window<TK, 2, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, ci, klist, sel->tmp);
+    else if (nch == 3) nw = select_window<TK, 3, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, ci, klist, sel->tmp);
+    else nw = select_window<TK, 4, CMB_THREADS>(a.x, a.I, a.k, tk, xs, sel, ci, klist, sel->tmp);
     u1 = (uint32_t)nw;
   } else if (FUSED) {
     // The kept set as a threshold (top-k: computed here; threshold mask:
     // given), then this CTA's kept channels of its range, numbered from 0.
+    const uint32_t rm = (uint32_t)(ci >> 32) & 0xFFFFu, rn = (uint32_t)(ci >> 48);
+    const int c0 = (int)((uint32_t)a.I * rm / rn), c1 = (int)((uint32_t)a.I * (rm + 1) / rn);
     int T = (int)a.tau_key, cut = -1;
     if (MODE == CMB_TOPK) select_threshold(xs, a.I, a.k, sel, &T, &cut);
     u1 = (uint32_t)thresh_compact(xs, c0, c1, T, cut, klist, nullptr, sel->wcnt);
+  }
+  if (FUSED) {
+    pr = (int)((ci >> 8) & 3u);
+    sr = (int)((ci >> 10) & 0x3FFFFFu);
   }
   const int nv = (int)(u1 - u0);
   // Generation of the grid barrier before this CTA arrives on it: read after
