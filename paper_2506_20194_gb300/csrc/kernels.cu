@@ -1287,8 +1287,8 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   if (thresh) a.k = 1 << 16;   // no rank space: cursors never wrap
   // Item split.  Items are the (problem, segment) runs of kept channels, in
   // order.  When every run can have CTAs of its own, runs get CTAs in
-  // proportion to their estimated bytes (record = mask + 2 bytes per expected
-  // non-zero) and no CTA spans two runs: a run boundary inside a CTA would
+  // proportion to their estimated cost (mostly the number of records, see
+  // below) and no CTA spans two runs: a run boundary inside a CTA would
   // cost a mid-stream flush of all its consumers' rows.  A CTA of a fused mode
   // takes a channel range of its run (the kept set is a threshold, so it can
   // find its own kept channels); with a kept list it takes a rank range.
@@ -1304,8 +1304,14 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
     int r = 0;
     for (int p = 0; p < a.np; ++p)
       for (int s = 0; s < a.p[p].S; ++s, ++r) {
+        // A run's cost: its k records, each one warp's walk over 1024 rows
+        // whatever the segment holds (a 768-row record measured 0.99 of a
+        // full one in the stream), plus its bytes: a short last segment
+        // (13824 rows: 512) weighed by bytes alone got 3 CTAs of 854
+        // records where the others had 5 or 6 of 427-512.
         const int rows = std::min(SEG_ROWS, a.p[p].O - s * SEG_ROWS);
-        w[r] = (double)MASK_BYTES + 2.0 * (double)a.p[p].dens * rows;
+        const double full = (double)MASK_BYTES + 2.0 * (double)a.p[p].dens * SEG_ROWS;
+        w[r] = 4.0 * full + (double)MASK_BYTES + 2.0 * (double)a.p[p].dens * rows;
         n[r] = 1;
       }
     for (int extra = grid - nruns; extra > 0; --extra) {
