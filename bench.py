@@ -929,7 +929,7 @@ def measure_stack(duo, synth, dev, workload, L=None, pw=None, px=50, reps=20, wa
            "peak_kind": peak_kind, "roofline_us_per_token": breq / (peak * 1e9) * 1e6,
            "dense_fp16_GB_per_token": dense_bytes / 1e9,
            "dense_roofline_us_per_token": dense_bytes / (peak * 1e9) * 1e6,
-           "packed_GB": packed / 1e9, "pack_seconds": pack_s, "launches_per_token": 4 * L,
+           "packed_GB": packed / 1e9, "pack_seconds": pack_s, "calls_per_token": 4 * L,
            "reps": reps, "clocks": clocks}
     if dense:
         def fd():

@@ -1320,6 +1320,27 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
         if (w[q] * n[best] > w[best] * n[q]) best = q;
       ++n[best];
     }
+    // A launch ends with its busiest CTA.  When whole CTAs per run leave it
+    // far above the mean (56 gate/up runs of a 70B layer on 152 CTAs: runs
+    // of 2 and 3 CTAs, 1.36x the mean), half the products per launch do
+    // better (28 runs: 5 or 6 CTAs, 1.09x) than one launch saves in
+    // selection and prologue.
+    if (a.np >= 2) {
+      double wsum = 0.0, wmax = 0.0;
+      for (int q = 0; q < nruns; ++q) {
+        wsum += w[q];
+        wmax = std::max(wmax, w[q] / n[q]);
+      }
+      if (wmax > 1.25 * wsum / grid) {
+        CmbArgs b0 = a0, b1 = a0;
+        const int h = a0.np / 2;
+        b0.np = h;
+        b1.np = a0.np - h;
+        for (int p = 0; p < b1.np; ++p) b1.p[p] = a0.p[h + p];
+        e = launch_cmb_spmspv(b0, st);
+        return e != cudaSuccess ? e : launch_cmb_spmspv(b1, st);
+      }
+    }
     a.run_cta[0] = 0;
     per_cta = 0;
     for (int q = 0; q < nruns; ++q) {
