@@ -1268,6 +1268,43 @@ __global__ void __launch_bounds__(CMB_THREADS, 1) cmb_spmspv_kernel(const CmbArg
   }
 }
 
+// Host: whole CTAs for each (product, segment) run of a launch (runs in
+// product order, at most kMaxRuns, at most grid of them) into n, greedily in
+// proportion to each run's estimated cost.  A run's cost is its k records,
+// each one warp's walk over 1024 rows whatever the segment holds (a 768-row
+// record measured 0.99 of a full one in the stream), plus its bytes: a short
+// last segment (13824 rows: 512) weighed by bytes alone got 3 CTAs of 854
+// records where the others had 5 or 6 of 427-512.  Returns true when the
+// launch should rather be two launches of half the products each: a launch
+// ends with its busiest CTA, and when whole CTAs per run leave that CTA far
+// above the mean (56 gate/up runs of a 70B layer on 152 CTAs: runs of 2 and
+// 3 CTAs, 1.36x the mean), half the products per launch do better (28 runs:
+// 5 or 6 CTAs, 1.09x) than one launch saves in selection and prologue.
+bool plan_runs(const CmbArgs& a, int grid, int* n) {
+  double w[kMaxRuns];
+  int nruns = 0;
+  for (int p = 0; p < a.np; ++p)
+    for (int s = 0; s < a.p[p].S; ++s, ++nruns) {
+      const int rows = std::min(SEG_ROWS, a.p[p].O - s * SEG_ROWS);
+      const double full = (double)MASK_BYTES + 2.0 * (double)a.p[p].dens * SEG_ROWS;
+      w[nruns] = 4.0 * full + (double)MASK_BYTES + 2.0 * (double)a.p[p].dens * rows;
+      n[nruns] = 1;
+    }
+  for (int extra = grid - nruns; extra > 0; --extra) {
+    int best = 0;
+    for (int q = 1; q < nruns; ++q)
+      if (w[q] * n[best] > w[best] * n[q]) best = q;
+    ++n[best];
+  }
+  if (a.np < 2) return false;
+  double wsum = 0.0, wmax = 0.0;
+  for (int q = 0; q < nruns; ++q) {
+    wsum += w[q];
+    wmax = std::max(wmax, w[q] / n[q]);
+  }
+  return wmax > 1.25 * wsum / grid;
+}
+
 cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   CmbArgs a = a0;
   if (a.wait_ns == 0) a.wait_ns = WAIT_LIMIT_NS;
@@ -1287,8 +1324,8 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   if (thresh) a.k = 1 << 16;   // no rank space: cursors never wrap
   // Item split.  Items are the (problem, segment) runs of kept channels, in
   // order.  When every run can have CTAs of its own, runs get CTAs in
-  // proportion to their estimated cost (mostly the number of records, see
-  // below) and no CTA spans two runs: a run boundary inside a CTA would
+  // proportion to their estimated cost (plan_runs: mostly the number of
+  // records) and no CTA spans two runs: a run boundary inside a CTA would
   // cost a mid-stream flush of all its consumers' rows.  A CTA of a fused mode
   // takes a channel range of its run (the kept set is a threshold, so it can
   // find its own kept channels); with a kept list it takes a rank range.
@@ -1299,47 +1336,15 @@ cudaError_t launch_cmb_spmspv(const CmbArgs& a0, cudaStream_t st) {
   int64_t per_cta = (total + grid - 1) / grid;
   a.nruns = 0;
   if (nruns <= kMaxRuns && nruns <= grid) {
-    double w[kMaxRuns];
     int n[kMaxRuns];
-    int r = 0;
-    for (int p = 0; p < a.np; ++p)
-      for (int s = 0; s < a.p[p].S; ++s, ++r) {
-        // A run's cost: its k records, each one warp's walk over 1024 rows
-        // whatever the segment holds (a 768-row record measured 0.99 of a
-        // full one in the stream), plus its bytes: a short last segment
-        // (13824 rows: 512) weighed by bytes alone got 3 CTAs of 854
-        // records where the others had 5 or 6 of 427-512.
-        const int rows = std::min(SEG_ROWS, a.p[p].O - s * SEG_ROWS);
-        const double full = (double)MASK_BYTES + 2.0 * (double)a.p[p].dens * SEG_ROWS;
-        w[r] = 4.0 * full + (double)MASK_BYTES + 2.0 * (double)a.p[p].dens * rows;
-        n[r] = 1;
-      }
-    for (int extra = grid - nruns; extra > 0; --extra) {
-      int best = 0;
-      for (int q = 1; q < nruns; ++q)
-        if (w[q] * n[best] > w[best] * n[q]) best = q;
-      ++n[best];
-    }
-    // A launch ends with its busiest CTA.  When whole CTAs per run leave it
-    // far above the mean (56 gate/up runs of a 70B layer on 152 CTAs: runs
-    // of 2 and 3 CTAs, 1.36x the mean), half the products per launch do
-    // better (28 runs: 5 or 6 CTAs, 1.09x) than one launch saves in
-    // selection and prologue.
-    if (a.np >= 2) {
-      double wsum = 0.0, wmax = 0.0;
-      for (int q = 0; q < nruns; ++q) {
-        wsum += w[q];
-        wmax = std::max(wmax, w[q] / n[q]);
-      }
-      if (wmax > 1.25 * wsum / grid) {
-        CmbArgs b0 = a0, b1 = a0;
-        const int h = a0.np / 2;
-        b0.np = h;
-        b1.np = a0.np - h;
-        for (int p = 0; p < b1.np; ++p) b1.p[p] = a0.p[h + p];
-        e = launch_cmb_spmspv(b0, st);
-        return e != cudaSuccess ? e : launch_cmb_spmspv(b1, st);
-      }
+    if (plan_runs(a, grid, n)) {   // two launches of half the products each
+      CmbArgs b0 = a0, b1 = a0;
+      const int h = a0.np / 2;
+      b0.np = h;
+      b1.np = a0.np - h;
+      for (int p = 0; p < b1.np; ++p) b1.p[p] = a0.p[h + p];
+      e = launch_cmb_spmspv(b0, st);
+      return e != cudaSuccess ? e : launch_cmb_spmspv(b1, st);
     }
     a.run_cta[0] = 0;
     per_cta = 0;
@@ -1473,6 +1478,35 @@ __global__ void __launch_bounds__(IDX16_THREADS, 1) idx16_spmspv_kernel(const Id
     }
   }
 }
+
+}  // namespace duo
+
+// Internal test entry point (not part of include/duo.h): the launcher's run
+// plan for np products of O[p] rows and density dens[p] on grid CTAs.  Host
+// only (no device call).  Writes each run's CTA count to n_out (runs in
+// product order; room for 128) and returns their number, with *split = 1
+// when the launch would be issued as two; -1 on bad arguments.
+extern "C" int duo_test_plan_runs(int np, const int* O, const float* dens, int grid, int* n_out,
+                                  int* split) {
+  if (np < 1 || np > duo::kMaxProblems || O == nullptr || dens == nullptr || n_out == nullptr ||
+      split == nullptr || grid < 1)
+    return -1;
+  duo::CmbArgs a{};
+  a.np = np;
+  int nruns = 0;
+  for (int p = 0; p < np; ++p) {
+    if (O[p] < 1) return -1;
+    a.p[p].O = O[p];
+    a.p[p].S = (O[p] + duo::SEG_ROWS - 1) / duo::SEG_ROWS;
+    a.p[p].dens = dens[p];
+    nruns += a.p[p].S;
+  }
+  if (nruns > duo::kMaxRuns || nruns > grid) return -1;
+  *split = duo::plan_runs(a, grid, n_out) ? 1 : 0;
+  return nruns;
+}
+
+namespace duo {
 
 cudaError_t launch_idx16_spmspv(const Idx16Args& a, cudaStream_t st) {
   DevProps dp;

@@ -75,6 +75,9 @@ def load_library(path: str | None = None):
     # internal, for the tensor-core GEMM's parity tests
     lib.duo_test_tc_gemm.argtypes = [i32, i32, i32, i32, i32, vp, i64, i64, i64, vp, i64, i64, i64, vp, i64, i64,
                                      i64, ctypes.c_float, ctypes.c_float, i32, i32, vp]
+    # internal, for the CPU test of the launcher's run plan
+    lib.duo_test_plan_runs.argtypes = [i32, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_float), i32,
+                                       ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_int)]
     lib.duo_copy.argtypes = [vp, vp, i64, vp]
     lib.duo_calib_create.argtypes = [i64, i64, vp, ctypes.POINTER(vp)]
     lib.duo_calib_precompute.argtypes = [vp, vp, i64, ctypes.c_float, i32, vp]
@@ -92,7 +95,7 @@ def load_library(path: str | None = None):
                  "duo_pack_cmb_noalloc", "duo_sparsify_threshold", "duo_spmspv_threshold",
                  "duo_calib_create", "duo_calib_precompute", "duo_calib_status", "duo_calib_export",
                  "duo_calib_score", "duo_calib_free", "duo_calib_prune", "duo_copy", "duo_calib_query",
-                 "duo_packed_status", "duo_test_spmspv_blocked", "duo_test_tc_gemm"):
+                 "duo_packed_status", "duo_test_spmspv_blocked", "duo_test_tc_gemm", "duo_test_plan_runs"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
