@@ -38,8 +38,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch of
 # the fused kernel from one ncu capture, valid only for the kernel source it
 # was taken on (sha256 of kernels.cu + duo_device.cuh, first 16 hex digits).
-TRAFFIC = {"sha": "f662772847820899",
-           "per_launch_bytes": [29113856.0, 9760512.0, 51907072.0, 26118144.0]}
+TRAFFIC = {"sha": "68c049807b7c2ca1",
+           "per_launch_bytes": [29113088.0, 9761024.0, 51911168.0, 26117632.0]}
 
 
 def parse():
